@@ -1,0 +1,385 @@
+#!/usr/bin/env python3
+"""Verify-step benchmark on the Llama-3.1-8B-shaped workload (batch 1, context
+2048, 32 query / 8 KV heads, head dim 128, hidden 4096, vocab 128256, 60-node
+EAGLE-style tree of depth <= 8 and top-k 10, tau = 0.3), synthetic seeded data.
+
+One step = the whole hot path through the C ABI (asd_verify_step): tree
+preparation, tree attention + split combine, the tcgen05 LM head with the
+fused margin epilogue, and the merge / accepted-path / K/V-commit tail.
+
+  python bench.py [--gpus N --steps K --warmup W] [--impl reference]
+
+Prints one JSON line.  Under torchrun every rank runs its own replica of the
+workload (weak scaling, no data-path collective); value = all ranks' nodes /
+the slowest rank's time.  `--impl reference` times the fp64 CPU oracle on a
+bounded sample instead (rank 0 only).
+"""
+import argparse
+import csv
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "verified tree nodes/s"
+UNIT = "nodes/s"
+CONFIG = 2
+TAU = 0.3
+N_STAGE_KERNELS = 5   # prep, attention, combine, LM head, tail
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=50)
+    ap.add_argument("--impl", default="asd", choices=["asd", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-clocks", action="store_true")
+    return ap.parse_args()
+
+
+def peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+def workload_config(wl):
+    return {
+        "workload": "llama3.1-8b-shaped verify step: batch 1, context 2048, 32 q / 8 kv heads, "
+                    "head_dim 128, hidden 4096, vocab 128256, 60-node EAGLE-style tree "
+                    "(depth<=8, top-k 10), tau 0.3, bf16",
+        "batch": wl.B, "ctx": int(wl.ctx_len[0]), "tree_nodes": wl.T,
+        "tree_depth": int(wl.max_path - 1), "tau": TAU,
+        "l2": "inputs larger than L2: the 1.05 GB LM-head weight is streamed every step",
+    }
+
+
+def lmhead_bytes(wl):
+    """Algorithmic bytes of the LM-head kernel: W and the hidden states read once,
+    per-row statistics written."""
+    return wl.vocab * wl.hidden_dim * 2 + wl.T * wl.hidden_dim * 2 + wl.T * 16
+
+
+def step_bytes(wl, mean_path):
+    """Algorithmic bytes of one verify step (every input read once, outputs written)."""
+    ctx = int(wl.ctx_len.sum())
+    attn = (ctx * wl.Hkv * wl.D * 2 * 2            # context K and V
+            + wl.T * wl.Hkv * wl.D * 2 * 2        # tree K and V
+            + wl.T * wl.Hq * wl.D * 2 * 2)        # Q read, O written
+    commit = mean_path * wl.B * wl.Hkv * wl.D * 2 * 2 * 2
+    return attn + lmhead_bytes(wl) + commit
+
+
+class Clocks:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index, enabled=True):
+        self.proc = None
+        self.path = None
+        if not enabled:
+            return
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(gpu_index), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        rows = []
+        with open(self.path) as f:
+            for r in csv.reader(f):
+                if len(r) >= 9:
+                    rows.append([x.strip() for x in r])
+        os.unlink(self.path)
+        if not rows:
+            return None
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({n for r in rows for n, v in zip(names, r[5:9]) if v.lower() == "active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": reasons, "samples": len(rows)}
+
+
+def ranks_torch(wl, device):
+    """Top-5 tokens of every parent row, for the drafted-token mixture (input
+    synthesis with a torch fp32 matmul on the device, outside any timing)."""
+    import torch
+    rows = wl.parents_needed()
+    h = torch.from_numpy(wl.hidden[rows]).to(device)
+    w = torch.from_numpy(wl.w).to(device=device, dtype=torch.bfloat16)
+    lg = torch.empty(len(rows), wl.vocab, device=device)
+    for v0 in range(0, wl.vocab, 16384):
+        lg[:, v0:v0 + 16384] = h @ w[v0:v0 + 16384].float().T
+    top = torch.topk(lg, 5, dim=1).indices.cpu().numpy()
+    del w, lg
+    return {int(r): top[j] for j, r in enumerate(rows)}
+
+
+def oracle_arrays(wl):
+    return dict(q=wl.q, k_cache=wl.k_cache, v_cache=wl.v_cache, ctx_len=wl.ctx_len,
+                tree_k=wl.tree_k, tree_v=wl.tree_v, parent=wl.parent, cu_nodes=wl.cu_nodes,
+                page_table=wl.page_table, page_size=wl.page_size, hidden=wl.hidden, w=wl.w,
+                tokens=wl.tokens)
+
+
+def cores_used():
+    try:
+        return len(os.sched_getaffinity(0))
+    except Exception:
+        return os.cpu_count()
+
+
+def cpu_baseline(wl, min_seconds=10.0):
+    """The oracle's whole verify step on the full workload, repeated until at
+    least `min_seconds` have passed (at most 3 repetitions)."""
+    import oracle
+    arrays = oracle_arrays(wl)
+    t0 = time.perf_counter()
+    reps = 0
+    while True:
+        oracle.verify_step(arrays, TAU)
+        reps += 1
+        el = time.perf_counter() - t0
+        if el >= min_seconds or reps >= 3:
+            break
+    return {"value": reps * wl.T / el, "unit": UNIT, "cores": cores_used(), "kind": "oracle",
+            "sample": f"{reps} full verify step(s) of the same workload ({wl.T} nodes, full vocab "
+                      f"and context) by the fp64 numpy oracle, {el:.1f} s"}
+
+
+def run_reference(args):
+    """The fp64 oracle as the reference arm, on a bounded sample per step."""
+    import oracle
+    from paper_2609_02897_gb300 import synth
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    full = synth.make_workload(CONFIG)
+    steps, warm = args.steps, args.warmup
+    budget = 120.0
+    target = budget / max(1, steps + warm)
+
+    def macs(wl):
+        anc = sum(len(oracle.ancestors_of(wl.parent, i)) for i in range(wl.T))
+        attn = 2 * wl.Hq * wl.D * (wl.T * int(wl.ctx_len[0]) + anc)
+        return attn + wl.T * wl.hidden_dim * wl.vocab
+
+    def sample(s):
+        wl = synth.make_workload(CONFIG, overrides=dict(vocab=max(64, full.vocab // s),
+                                                        ctx=(max(16, 2048 // s),) * 2))
+        rows = wl.parents_needed()
+        top = oracle.topk_tokens(wl.hidden, wl.w, rows, 5)
+        synth.attach_tokens(wl, {int(r): top[j] for j, r in enumerate(rows)})
+        return wl
+
+    s = 64
+    wl = sample(s)
+    t0 = time.perf_counter()
+    oracle.verify_step(oracle_arrays(wl), TAU)
+    t1 = time.perf_counter() - t0
+    s = int(min(4096, max(1, 2 ** round(np.log2(max(1e-9, s * t1 / target))))))
+    wl = sample(s)
+    arrays = oracle_arrays(wl)
+    for _ in range(warm):
+        oracle.verify_step(arrays, TAU)
+    t0 = time.perf_counter()
+    for _ in range(steps):
+        oracle.verify_step(arrays, TAU)
+    el = time.perf_counter() - t0
+    frac = macs(wl) / macs(full)
+    value = full.T * frac / (el / steps)
+    desc = (f"each step: the oracle's full verify step on the same tree and heads with the "
+            f"vocabulary cut to {wl.vocab} rows and the context to {int(wl.ctx_len[0])} tokens "
+            f"({frac:.2e} of the workload's multiply-adds); value scaled by that fraction")
+    print(json.dumps({
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": steps, "warmup": warm, "ms_per_step": 1e3 * el / steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": workload_config(full),
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores_used(), "kind": "oracle",
+                         "sample": desc},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }))
+
+
+def run_asd(args):
+    import torch
+    import torch.distributed as dist
+
+    from paper_2609_02897_gb300 import asd, synth
+
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    device = f"cuda:{local}"
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device(device))
+
+    wl = synth.make_workload(CONFIG, rep=rank)
+    synth.attach_tokens(wl, ranks_torch(wl, device))
+    bf = torch.bfloat16
+
+    def f(x):
+        return torch.from_numpy(np.ascontiguousarray(x)).to(device=device, dtype=bf)
+
+    def i(x):
+        return torch.from_numpy(np.ascontiguousarray(x, dtype=np.int32)).to(device)
+
+    inputs = dict(q=f(wl.q), tree_k=f(wl.tree_k), tree_v=f(wl.tree_v), hidden=f(wl.hidden),
+                  tokens=i(wl.tokens), parent=i(wl.parent), cu_nodes=i(wl.cu_nodes),
+                  ctx_len=i(wl.ctx_len))
+    w_lm = f(wl.w)
+    k_cache, v_cache = f(wl.k_cache), f(wl.v_cache)
+    dims = asd.make_dims(wl.B, wl.Hq, wl.Hkv, wl.D, wl.hidden_dim, wl.vocab, asd.ASD_BF16, 0,
+                         wl.ctx_max, 0, wl.T, wl.max_path)
+    step = asd.VerifyStep(dims, wl.T, device=device)
+    step.bind(w_lm=w_lm, k_cache=k_cache, v_cache=v_cache, tau=TAU, **inputs)
+    stream = torch.cuda.current_stream()
+
+    K, W = args.steps, args.warmup
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(K)]
+    for row in evs:
+        for e in row:
+            e.record(stream)   # creates the underlying CUDA events
+    t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+
+    clocks = Clocks(local, enabled=not args.no_clocks)
+    for _ in range(W):
+        step.run(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    t_start.record(stream)
+    for k in range(K):
+        for j in range(5):
+            step.args.stage_events[j] = evs[k][j].cuda_event
+        step.run(stream)
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    status = step.device_status()
+    if status != 0:
+        raise RuntimeError(f"device status {asd.STATUS.get(status, status)}")
+    ms = t_start.elapsed_time(t_end) / K
+    stage = np.array([[evs[k][j].elapsed_time(evs[k][j + 1]) for j in range(4)] for k in range(K)])
+    stage_ms = stage.mean(axis=0)
+    lm_ms = float(stage_ms[2])
+    if world > 1:
+        t = torch.tensor([ms, lm_ms], device=device, dtype=torch.float64)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms, lm_ms_max = float(t[0]), float(t[1])
+    mean_path = float(step.out["path_len"].float().mean())
+
+    # end to end through the public API: per step, H2D of the step's inputs
+    # from pinned host memory, the verify step, D2H of its results, host sync
+    e2e = None
+    if not args.no_e2e:
+        host_in = {k: v.cpu().pin_memory() for k, v in inputs.items()}
+        out_names = ["path", "path_len", "bonus", "n_promoted", "ctx_len_out", "accept", "row_lse"]
+        host_out = {k: torch.empty_like(step.out[k], device="cpu").pin_memory() for k in out_names}
+        h2d = sum(v.numel() * v.element_size() for v in host_in.values())
+        d2h = sum(v.numel() * v.element_size() for v in host_out.values())
+        for j in range(5):
+            step.args.stage_events[j] = None
+        for _ in range(min(W, 20)):
+            for k2, v in host_in.items():
+                inputs[k2].copy_(v, non_blocking=True)
+            step.run(stream)
+            for k2, v in host_out.items():
+                v.copy_(step.out[k2], non_blocking=True)
+            stream.synchronize()
+        if world > 1:
+            dist.barrier()
+        t0 = time.perf_counter()
+        for _ in range(K):
+            for k2, v in host_in.items():
+                inputs[k2].copy_(v, non_blocking=True)
+            step.run(stream)
+            for k2, v in host_out.items():
+                v.copy_(step.out[k2], non_blocking=True)
+            stream.synchronize()
+        e2e_s = (time.perf_counter() - t0) / K
+        if world > 1:
+            t = torch.tensor([e2e_s], device=device, dtype=torch.float64)
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            e2e_s = float(t[0])
+        e2e = {"value": world * wl.T / e2e_s, "unit": UNIT, "h2d_bytes_per_step": h2d,
+               "d2h_bytes_per_step": d2h, "us_per_step": 1e6 * e2e_s}
+
+    if rank != 0:
+        if world > 1:
+            dist.destroy_process_group()
+        return
+    peak, peak_kind = peaks()
+    lmb = lmhead_bytes(wl)
+    achieved = lmb / (lm_ms * 1e-3) / 1e9
+    sb = step_bytes(wl, mean_path)
+    line = {
+        "metric": METRIC, "value": world * wl.T / (ms * 1e-3), "unit": UNIT, "n_gpus": world,
+        "steps": K, "warmup": W, "ms_per_step": ms, "us_per_step": 1e3 * ms,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic (seeded; Llama-3.1-8B-shaped tensors, random weights)",
+        "config": workload_config(wl),
+        "hbm_gbs": sb / (ms * 1e-3) / 1e9, "hbm_frac_of_" + peak_kind: sb / (ms * 1e-3) / 1e9 / peak,
+        "roofline": {"kernel": "lmhead_tc_kernel", "bound": "hbm", "achieved": achieved,
+                     "peak": peak, "unit": "GB/s", "frac": achieved / peak,
+                     "peak_source": peak_kind + " hbm_gbs (MEASURED_PEAKS.json)",
+                     "algorithmic_bytes_per_launch": lmb, "avg_launch_us": 1e3 * lm_ms,
+                     "traffic": None},
+        "stages_us": {"prep": 1e3 * stage_ms[0], "attention+combine": 1e3 * stage_ms[1],
+                      "lmhead": 1e3 * stage_ms[2], "tail": 1e3 * stage_ms[3]},
+        "mean_path_len": mean_path,
+        "gpu_launches": K * N_STAGE_KERNELS,
+        "clocks": clk,
+        "e2e": e2e,
+    }
+    if world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(wl)
+    print(json.dumps(line))
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_asd(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,230 @@
+/*
+ * asd.h - C ABI of libasd: the per-step tree-verification path of margin-based
+ * lossy speculative decoding ("Margins, Not Windows: Training-Free Per-Step
+ * Lossy Speculative Decoding", arXiv 2609.02897) on one NVIDIA GB300 (sm_103a).
+ *
+ * One verify step (Sec. 2 "Verify", Sec. 3.1-3.2) takes a draft tree of N nodes
+ * per sequence - node 0 is the root (the last committed token, whose K/V is not
+ * yet in the cache), nodes 1..N-1 carry drafted tokens - and
+ *   1. runs the target's attention for every node over the committed context
+ *      plus the node's tree ancestors (asd_tree_attention);
+ *   2. projects the node hidden states through the LM head and, without
+ *      writing logits to memory, reduces every row to its max, argmax and
+ *      log-sum-exp and evaluates the margin rule of Eq. 1 for every drafted
+ *      token (asd_lmhead_margin);
+ *   3. picks the longest root-to-node path of accepted nodes (asd_accept_path);
+ *   4. appends the K/V of that path to the cache (asd_kv_compact).
+ * asd_verify_step chains the four on one stream.
+ *
+ * Conventions shared by every call
+ *  - All tensor arguments are DEVICE pointers owned by the caller; the library
+ *    never allocates, frees or keeps pointers after a call returns.  Every
+ *    call only enqueues work on `stream` (a cudaStream_t passed as void*; NULL
+ *    is the legacy default stream) and returns without synchronising, so a
+ *    sequence of calls can be captured in a CUDA graph.
+ *  - Sequences are packed: cu_nodes[B+1] (int32, cu_nodes[0] = 0) delimits the
+ *    nodes of each sequence in every [T, ...] array, T = cu_nodes[B] =
+ *    total_nodes.  parent[T] holds LOCAL parent ids: parent[root] = -1 and
+ *    0 <= parent[i] < i for the other nodes (topological numbering).  At most
+ *    ASD_MAX_TREE_NODES nodes per sequence.
+ *  - Row-major layouts, innermost dimension last.  Element type of q, caches,
+ *    tree K/V, hidden, W and the attention output: dims->dtype (fp32 or bf16).
+ *    Tensors read through TMA (caches, hidden, W) must be 16-byte aligned.
+ *  - tau is the paper's margin threshold kappa (Eq. 1 and the rule after it),
+ *    0 < tau <= 1.  The rule is evaluated as l_draft - row_max >= ln(tau) with
+ *    ln(tau) computed on the host in double precision.
+ *  - Errors: arguments that the host can check (null pointers, dims, tau,
+ *    workspace size) make a call return a non-OK status before anything is
+ *    enqueued.  Errors that only the device can see (malformed parent array,
+ *    token id outside [0, vocab), ctx_len beyond the cache, a page id outside
+ *    the pool, a path longer than max_path, a bounded wait that gave up) are
+ *    recorded as the FIRST error code in the workspace status word and the
+ *    affected sequence gets path_len = 0 and no cache write; kernels never
+ *    trap.  Every call that takes a workspace clears its status word first;
+ *    asd_get_device_status reads it.  Launch failures return ASD_ERR_CUDA.
+ */
+#ifndef ASD_H_
+#define ASD_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define ASD_ABI_VERSION 1
+#define ASD_MAX_TREE_NODES 128
+#define ASD_NUM_STAGE_EVENTS 5
+
+typedef enum asd_status {
+  ASD_OK = 0,
+  ASD_ERR_INVALID_ARG = 1, /* null pointer, bad enum, tau outside (0, 1]       */
+  ASD_ERR_SHAPE = 2,       /* dims inconsistent or unsupported; path too long   */
+  ASD_ERR_TREE = 3,        /* device: malformed parent array or cu_nodes        */
+  ASD_ERR_TOKEN_RANGE = 4, /* device: drafted token id outside [0, vocab)       */
+  ASD_ERR_CTX_RANGE = 5,   /* device: ctx_len beyond the cache / bad page id    */
+  ASD_ERR_WORKSPACE = 6,   /* workspace too small or misaligned                 */
+  ASD_ERR_CUDA = 7,        /* a CUDA runtime/driver call or launch failed       */
+  ASD_ERR_TIMEOUT = 8,     /* device: a bounded wait inside a kernel gave up    */
+  ASD_ERR_UNSUPPORTED = 9  /* device is not sm_103 / feature not built          */
+} asd_status;
+
+typedef enum asd_dtype { ASD_F32 = 0, ASD_BF16 = 1 } asd_dtype;
+
+/* Shapes of one verify step.  All fields are int32. */
+typedef struct asd_dims {
+  int32_t batch;        /* B: number of sequences (trees)                      */
+  int32_t num_q_heads;  /* Hq                                                  */
+  int32_t num_kv_heads; /* Hkv; Hq % Hkv == 0 (grouped-query attention)        */
+  int32_t head_dim;     /* D: 64 or 128                                        */
+  int32_t hidden;       /* LM-head input width (multiple of 8)                 */
+  int32_t vocab;        /* V: LM-head rows                                     */
+  int32_t dtype;        /* asd_dtype                                           */
+  int32_t page_size;    /* 0: contiguous cache; else tokens per page, a power
+                           of two in [8, 256]                                  */
+  int32_t ctx_max;      /* cache slots per sequence: contiguous capacity, or
+                           (page-table columns) * page_size when paged         */
+  int32_t num_pages;    /* P: pages in the pool (paged), else 0                */
+  int32_t max_nodes;    /* upper bound on nodes per tree, 1..128               */
+  int32_t max_path;     /* columns of the path output, >= longest root-to-leaf
+                           path (nodes, root included)                         */
+} asd_dims;
+
+/* Bytes of device workspace that the calls below need for `total_nodes`
+ * nodes with these dims on the current device (depends on its SM count).
+ * Returns 0 if the dims are invalid.  The workspace needs no initialisation;
+ * its address must be 256-byte aligned. */
+size_t asd_workspace_bytes(const asd_dims* dims, int32_t total_nodes);
+
+/*
+ * Tree attention (step 1; Sec. 2 "Verify", Sec. 3.1: the target scores all
+ * drafted nodes in one forward pass).
+ * For node i of sequence b and query head h (KV head g = h / (Hq/Hkv)):
+ *   keys   = context positions 0..ctx_len[b]-1, then the tree ancestors of i
+ *            from the root down to i itself;
+ *   out[i,h] = softmax_j(q[i,h] . k_j / sqrt(D)) . v_j      (fp32 softmax)
+ *  q       [T, Hq, D]
+ *  k_cache, v_cache: contiguous [B, Hkv, ctx_max, D], or paged pool
+ *            [P, Hkv, page_size, D] addressed through
+ *  page_table [B, ctx_max / page_size] int32 (NULL when contiguous)
+ *  ctx_len [B] int32, 0 <= ctx_len[b] <= ctx_max
+ *  tree_k, tree_v [T, Hkv, D]: the K/V of the tree nodes themselves
+ *  out     [T, Hq, D] (dtype of the inputs)
+ * q and K are taken as given (positions already applied).
+ */
+asd_status asd_tree_attention(const asd_dims* dims, const void* q, const void* k_cache,
+                              const void* v_cache, const int32_t* page_table,
+                              const int32_t* ctx_len, const void* tree_k, const void* tree_v,
+                              const int32_t* parent, const int32_t* cu_nodes,
+                              int32_t total_nodes, void* out, void* workspace,
+                              size_t workspace_bytes, void* stream);
+
+/*
+ * LM head fused with the margin rule (step 2; Eq. 1 and the kappa rule).
+ * logits[i,v] = sum_k hidden[i,k] * w_lm[v,k]  (fp32 accumulation; never stored)
+ *  hidden [T, hidden], w_lm [V, hidden] (HF lm_head.weight layout),
+ *  tokens [T] int32: drafted token of each node (the root's is ignored).
+ * Per row i:  row_max[i], row_argmax[i] (lowest index attaining the max),
+ *             row_lse[i] = row_max + ln sum_v exp(logit - row_max).
+ * Per non-root node c with parent p:  l_draft[c] = logits[p, tokens[c]],
+ *             ratio[c] = exp(l_draft[c] - row_max[p])  (Eq. 1),
+ *             accept[c] = tokens[c] == row_argmax[p]  ||  ratio >= tau.
+ * Roots: accept = 1, l_draft = ratio = NaN.  Outputs are [T] arrays
+ * (float32 / int32 / uint8).
+ */
+asd_status asd_lmhead_margin(const asd_dims* dims, const void* hidden, const void* w_lm,
+                             const int32_t* tokens, const int32_t* parent,
+                             const int32_t* cu_nodes, int32_t total_nodes, float tau,
+                             float* row_max, int32_t* row_argmax, float* row_lse,
+                             float* l_draft, float* ratio, uint8_t* accept, void* workspace,
+                             size_t workspace_bytes, void* stream);
+
+/*
+ * Accepted path (step 3; Sec. 3.2 and Fig. 1: verification commits the
+ * drafted tokens up to the first node that is neither a strict match nor
+ * promoted by the margin rule).  Over the tree this is the longest root-to-
+ * node path whose non-root nodes all have accept = 1; equally long paths are
+ * ordered by their node-index sequences and the smallest wins.
+ *  accept [T] uint8, row_argmax [T] int32, tokens [T] int32 (inputs)
+ *  path [B, max_path] int32: local node ids, root first, -1 padded
+ *  path_len [B]: nodes on the path including the root (>= 1)
+ *  bonus [B]: row_argmax of the last path node (the next committed token)
+ *  n_promoted [B]: path nodes whose token is not the parent row's argmax
+ */
+asd_status asd_accept_path(const asd_dims* dims, const int32_t* parent, const int32_t* tokens,
+                           const uint8_t* accept, const int32_t* row_argmax,
+                           const int32_t* cu_nodes, int32_t total_nodes, int32_t* path,
+                           int32_t* path_len, int32_t* bonus, int32_t* n_promoted,
+                           void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * K/V commit of the accepted path (step 4; Sec. 2: the accepted tokens are
+ * committed after one target pass).  For k < path_len[b], the K and V rows
+ * (all Hkv heads) of tree node path[b,k] go to cache slot ctx_len[b] + k of
+ * sequence b - in place in a contiguous cache, or through page_table (whose
+ * columns past the context must already name fresh pages) when paged.
+ * ctx_len_out[b] = ctx_len[b] + path_len[b].  Tree K/V and cache never alias.
+ */
+asd_status asd_kv_compact(const asd_dims* dims, const void* tree_k, const void* tree_v,
+                          const int32_t* cu_nodes, int32_t total_nodes, const int32_t* path,
+                          const int32_t* path_len, const int32_t* ctx_len,
+                          const int32_t* page_table, void* k_cache, void* v_cache,
+                          int32_t* ctx_len_out, void* workspace, size_t workspace_bytes,
+                          void* stream);
+
+/* Arguments of asd_verify_step: the union of the four calls above. */
+typedef struct asd_verify_args {
+  /* inputs */
+  const void* q;
+  const void* tree_k;
+  const void* tree_v;
+  const void* hidden;
+  const void* w_lm;
+  const int32_t* tokens;
+  const int32_t* parent;
+  const int32_t* cu_nodes;
+  const int32_t* ctx_len;
+  const int32_t* page_table; /* NULL when contiguous                          */
+  int32_t total_nodes;
+  float tau;
+  /* read by attention, appended to by the commit (disjoint slots)         */
+  void* k_cache;
+  void* v_cache;
+  /* outputs */
+  void* attn_out;
+  float* row_max;
+  int32_t* row_argmax;
+  float* row_lse;
+  float* l_draft;
+  float* ratio;
+  uint8_t* accept;
+  int32_t* path;
+  int32_t* path_len;
+  int32_t* bonus;
+  int32_t* n_promoted;
+  int32_t* ctx_len_out;
+  /* optional cudaEvent_t handles (NULL to skip), recorded on `stream` at:
+     [0] start, [1] after tree preparation, [2] after attention,
+     [3] after the LM-head GEMM kernel, [4] after path choice and commit. */
+  void* stage_events[ASD_NUM_STAGE_EVENTS];
+} asd_verify_args;
+
+/* One whole verify step, steps 1-4 on one stream (same semantics as the
+ * individual calls; attention reads only the slots below ctx_len, the commit
+ * writes only slots at or above it). */
+asd_status asd_verify_step(const asd_dims* dims, const asd_verify_args* args, void* workspace,
+                           size_t workspace_bytes, void* stream);
+
+/* Copies the workspace status word (first device-side error of the most
+ * recent call, ASD_OK if none) to *status_out.  Synchronises `stream`. */
+asd_status asd_get_device_status(const void* workspace, int32_t* status_out, void* stream);
+
+const char* asd_status_string(int32_t status);
+int32_t asd_abi_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* ASD_H_ */

@@ -63,9 +63,9 @@ def tree_attention(q, k_cache, v_cache, ctx_len, tree_k, tree_v, parent, cu_node
                 anc = [s + a for a in ancestors_of(par, i)]
                 keys = np.concatenate([kc, np.asarray(tree_k[anc, g], dtype=np.float64)])
                 vals = np.concatenate([vc, np.asarray(tree_v[anc, g], dtype=np.float64)])
-                for h in range(g * G, (g + 1) * G):
-                    sc = keys @ q[t, h] * scale
-                    p = np.exp(sc - sc.max())
-                    p /= p.sum()
-                    out[t, h] = p @ vals
+                # the G query heads that share KV head g, one softmax row each
+                sc = q[t, g * G:(g + 1) * G] @ keys.T * scale
+                p = np.exp(sc - sc.max(axis=1, keepdims=True))
+                p /= p.sum(axis=1, keepdims=True)
+                out[t, g * G:(g + 1) * G] = p @ vals
     return out

@@ -1,0 +1,232 @@
+"""ctypes binding of libasd (include/asd.h).  Argument marshalling only: every
+step of the verify path runs in the library's CUDA kernels.  Tensors are torch
+tensors used as device memory; the stream defaults to torch's current stream.
+
+Importing this module loads libasd.so and raises ImportError if it has not
+been built (paper_2609_02897_gb300.build.build()).  There is no fallback.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Optional, Sequence
+
+import torch
+
+_LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "_lib", "libasd.so")
+if not os.path.exists(_LIB_PATH):
+    raise ImportError(f"libasd is not built ({_LIB_PATH} missing); run "
+                      "`python -c 'import __graft_entry__ as g; g.build()'`")
+_lib = ctypes.CDLL(_LIB_PATH)
+
+ASD_F32, ASD_BF16 = 0, 1
+MAX_TREE_NODES = 128
+NUM_STAGE_EVENTS = 5
+STATUS = {0: "ASD_OK", 1: "ASD_ERR_INVALID_ARG", 2: "ASD_ERR_SHAPE", 3: "ASD_ERR_TREE",
+          4: "ASD_ERR_TOKEN_RANGE", 5: "ASD_ERR_CTX_RANGE", 6: "ASD_ERR_WORKSPACE",
+          7: "ASD_ERR_CUDA", 8: "ASD_ERR_TIMEOUT", 9: "ASD_ERR_UNSUPPORTED"}
+EXPORTS = ["asd_workspace_bytes", "asd_tree_attention", "asd_lmhead_margin", "asd_accept_path",
+           "asd_kv_compact", "asd_verify_step", "asd_get_device_status", "asd_status_string",
+           "asd_abi_version"]
+
+
+class AsdError(RuntimeError):
+    def __init__(self, code: int, where: str):
+        self.code = code
+        super().__init__(f"{where}: {STATUS.get(code, code)} "
+                         f"({_lib.asd_status_string(code).decode()})")
+
+
+class Dims(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_int32) for n in (
+        "batch", "num_q_heads", "num_kv_heads", "head_dim", "hidden", "vocab", "dtype",
+        "page_size", "ctx_max", "num_pages", "max_nodes", "max_path")]
+
+
+_vp = ctypes.c_void_p
+_i32p = ctypes.c_void_p
+
+
+class VerifyArgs(ctypes.Structure):
+    _fields_ = [
+        ("q", _vp), ("tree_k", _vp), ("tree_v", _vp), ("hidden", _vp), ("w_lm", _vp),
+        ("tokens", _vp), ("parent", _vp), ("cu_nodes", _vp), ("ctx_len", _vp),
+        ("page_table", _vp), ("total_nodes", ctypes.c_int32), ("tau", ctypes.c_float),
+        ("k_cache", _vp), ("v_cache", _vp),
+        ("attn_out", _vp), ("row_max", _vp), ("row_argmax", _vp), ("row_lse", _vp),
+        ("l_draft", _vp), ("ratio", _vp), ("accept", _vp), ("path", _vp), ("path_len", _vp),
+        ("bonus", _vp), ("n_promoted", _vp), ("ctx_len_out", _vp),
+        ("stage_events", _vp * NUM_STAGE_EVENTS),
+    ]
+
+
+_P = ctypes.POINTER(Dims)
+_lib.asd_abi_version.restype = ctypes.c_int32
+_lib.asd_status_string.restype = ctypes.c_char_p
+_lib.asd_status_string.argtypes = [ctypes.c_int32]
+_lib.asd_workspace_bytes.restype = ctypes.c_size_t
+_lib.asd_workspace_bytes.argtypes = [_P, ctypes.c_int32]
+_lib.asd_tree_attention.restype = ctypes.c_int
+_lib.asd_tree_attention.argtypes = [_P] + [_vp] * 9 + [ctypes.c_int32, _vp, _vp, ctypes.c_size_t, _vp]
+_lib.asd_lmhead_margin.restype = ctypes.c_int
+_lib.asd_lmhead_margin.argtypes = [_P] + [_vp] * 5 + [ctypes.c_int32, ctypes.c_float] + [_vp] * 6 + [
+    _vp, ctypes.c_size_t, _vp]
+_lib.asd_accept_path.restype = ctypes.c_int
+_lib.asd_accept_path.argtypes = [_P] + [_vp] * 5 + [ctypes.c_int32] + [_vp] * 4 + [
+    _vp, ctypes.c_size_t, _vp]
+_lib.asd_kv_compact.restype = ctypes.c_int
+_lib.asd_kv_compact.argtypes = [_P, _vp, _vp, _vp, ctypes.c_int32] + [_vp] * 7 + [
+    _vp, ctypes.c_size_t, _vp]
+_lib.asd_verify_step.restype = ctypes.c_int
+_lib.asd_verify_step.argtypes = [_P, ctypes.POINTER(VerifyArgs), _vp, ctypes.c_size_t, _vp]
+_lib.asd_get_device_status.restype = ctypes.c_int
+_lib.asd_get_device_status.argtypes = [_vp, ctypes.POINTER(ctypes.c_int32), _vp]
+
+
+def lib_path() -> str:
+    return _LIB_PATH
+
+
+def abi_version() -> int:
+    return int(_lib.asd_abi_version())
+
+
+def make_dims(batch, num_q_heads, num_kv_heads, head_dim, hidden, vocab, dtype, page_size,
+              ctx_max, num_pages, max_nodes, max_path) -> Dims:
+    return Dims(batch, num_q_heads, num_kv_heads, head_dim, hidden, vocab, dtype, page_size,
+                ctx_max, num_pages, max_nodes, max_path)
+
+
+def _ptr(t: Optional[torch.Tensor]):
+    if t is None:
+        return None
+    if not t.is_cuda:
+        raise ValueError("libasd takes device tensors")
+    if not t.is_contiguous():
+        raise ValueError("libasd takes contiguous tensors")
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream) -> ctypes.c_void_p:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream))
+
+
+def _check(code: int, where: str):
+    if code != 0:
+        raise AsdError(code, where)
+
+
+def asd_workspace_bytes(dims: Dims, total_nodes: int) -> int:
+    n = int(_lib.asd_workspace_bytes(ctypes.byref(dims), int(total_nodes)))
+    if n == 0:
+        raise AsdError(2, "asd_workspace_bytes")
+    return n
+
+
+def alloc_workspace(dims: Dims, total_nodes: int, device="cuda") -> torch.Tensor:
+    return torch.empty(asd_workspace_bytes(dims, total_nodes), dtype=torch.uint8, device=device)
+
+
+def asd_tree_attention(dims, q, k_cache, v_cache, page_table, ctx_len, tree_k, tree_v, parent,
+                       cu_nodes, out, workspace, stream=None):
+    _check(_lib.asd_tree_attention(
+        ctypes.byref(dims), _ptr(q), _ptr(k_cache), _ptr(v_cache), _ptr(page_table),
+        _ptr(ctx_len), _ptr(tree_k), _ptr(tree_v), _ptr(parent), _ptr(cu_nodes),
+        int(parent.numel()), _ptr(out), _ptr(workspace), workspace.numel(), _stream(stream)),
+        "asd_tree_attention")
+
+
+def asd_lmhead_margin(dims, hidden, w_lm, tokens, parent, cu_nodes, tau, row_max, row_argmax,
+                      row_lse, l_draft, ratio, accept, workspace, stream=None):
+    _check(_lib.asd_lmhead_margin(
+        ctypes.byref(dims), _ptr(hidden), _ptr(w_lm), _ptr(tokens), _ptr(parent), _ptr(cu_nodes),
+        int(parent.numel()), float(tau), _ptr(row_max), _ptr(row_argmax), _ptr(row_lse),
+        _ptr(l_draft), _ptr(ratio), _ptr(accept), _ptr(workspace), workspace.numel(),
+        _stream(stream)), "asd_lmhead_margin")
+
+
+def asd_accept_path(dims, parent, tokens, accept, row_argmax, cu_nodes, path, path_len, bonus,
+                    n_promoted, workspace, stream=None):
+    _check(_lib.asd_accept_path(
+        ctypes.byref(dims), _ptr(parent), _ptr(tokens), _ptr(accept), _ptr(row_argmax),
+        _ptr(cu_nodes), int(parent.numel()), _ptr(path), _ptr(path_len), _ptr(bonus),
+        _ptr(n_promoted), _ptr(workspace), workspace.numel(), _stream(stream)),
+        "asd_accept_path")
+
+
+def asd_kv_compact(dims, tree_k, tree_v, cu_nodes, total_nodes, path, path_len, ctx_len,
+                   page_table, k_cache, v_cache, ctx_len_out, workspace, stream=None):
+    _check(_lib.asd_kv_compact(
+        ctypes.byref(dims), _ptr(tree_k), _ptr(tree_v), _ptr(cu_nodes), int(total_nodes),
+        _ptr(path), _ptr(path_len), _ptr(ctx_len), _ptr(page_table), _ptr(k_cache),
+        _ptr(v_cache), _ptr(ctx_len_out), _ptr(workspace), workspace.numel(), _stream(stream)),
+        "asd_kv_compact")
+
+
+def asd_verify_step(dims, args: VerifyArgs, workspace, stream=None):
+    _check(_lib.asd_verify_step(ctypes.byref(dims), ctypes.byref(args), _ptr(workspace),
+                                workspace.numel(), _stream(stream)), "asd_verify_step")
+
+
+def asd_get_device_status(workspace, stream=None) -> int:
+    out = ctypes.c_int32(-1)
+    _check(_lib.asd_get_device_status(_ptr(workspace), ctypes.byref(out), _stream(stream)),
+           "asd_get_device_status")
+    return int(out.value)
+
+
+class VerifyStep:
+    """Owns the output tensors of one verify-step shape and the argument block.
+
+    Inputs are bound once (`bind`); `run()` enqueues asd_verify_step on the
+    stream.  `events` (optional list of 5 torch.cuda.Event with timing) are
+    recorded at the stage boundaries documented in asd.h.
+    """
+
+    OUT_FIELDS = ("attn_out", "row_max", "row_argmax", "row_lse", "l_draft", "ratio", "accept",
+                  "path", "path_len", "bonus", "n_promoted", "ctx_len_out")
+
+    def __init__(self, dims: Dims, total_nodes: int, device="cuda", attn_dtype=torch.bfloat16):
+        self.dims = dims
+        self.T = int(total_nodes)
+        T, B = self.T, dims.batch
+        f32 = dict(dtype=torch.float32, device=device)
+        i32 = dict(dtype=torch.int32, device=device)
+        self.out = dict(
+            attn_out=torch.empty(T, dims.num_q_heads, dims.head_dim, dtype=attn_dtype, device=device),
+            row_max=torch.empty(T, **f32), row_argmax=torch.empty(T, **i32),
+            row_lse=torch.empty(T, **f32), l_draft=torch.empty(T, **f32),
+            ratio=torch.empty(T, **f32), accept=torch.empty(T, dtype=torch.uint8, device=device),
+            path=torch.empty(B, dims.max_path, **i32), path_len=torch.empty(B, **i32),
+            bonus=torch.empty(B, **i32), n_promoted=torch.empty(B, **i32),
+            ctx_len_out=torch.empty(B, **i32))
+        self.workspace = alloc_workspace(dims, T, device)
+        self.args = VerifyArgs()
+        self._keep = []
+
+    def bind(self, *, q, tree_k, tree_v, hidden, w_lm, tokens, parent, cu_nodes, ctx_len,
+             k_cache, v_cache, tau, page_table=None, events: Optional[Sequence] = None):
+        a = self.args
+        self._keep = [q, tree_k, tree_v, hidden, w_lm, tokens, parent, cu_nodes, ctx_len,
+                      k_cache, v_cache, page_table]
+        a.q, a.tree_k, a.tree_v = _ptr(q), _ptr(tree_k), _ptr(tree_v)
+        a.hidden, a.w_lm, a.tokens = _ptr(hidden), _ptr(w_lm), _ptr(tokens)
+        a.parent, a.cu_nodes, a.ctx_len = _ptr(parent), _ptr(cu_nodes), _ptr(ctx_len)
+        a.page_table = _ptr(page_table)
+        a.total_nodes = self.T
+        a.tau = float(tau)
+        a.k_cache, a.v_cache = _ptr(k_cache), _ptr(v_cache)
+        for f in self.OUT_FIELDS:
+            setattr(a, f, _ptr(self.out[f]))
+        for i in range(NUM_STAGE_EVENTS):
+            a.stage_events[i] = (events[i].cuda_event if events is not None else None)
+        return self
+
+    def run(self, stream=None):
+        asd_verify_step(self.dims, self.args, self.workspace, stream)
+        return self.out
+
+    def device_status(self, stream=None) -> int:
+        return asd_get_device_status(self.workspace, stream)

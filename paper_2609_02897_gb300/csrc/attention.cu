@@ -1,0 +1,561 @@
+// Tree attention of the verify pass (Sec. 2 "Verify": the target scores every
+// drafted node of the tree in one forward pass).
+//
+// Work unit: one CTA per (row block, sequence x KV head, split).  The query
+// rows of a (sequence, KV head) pair are its N nodes times the G query heads
+// that share the KV head (grouped-query attention), packed node-major:
+// row r -> node r / G, head g*G + r % G.  Splits 0..n_splits-1 cover slices of
+// the committed context (flash-decoding split-KV); split n_splits covers the
+// tree itself, where a node only sees its ancestors (bitmask from the tree
+// preparation kernel).  Each split writes its softmax-normalised partial
+// output and its log-sum-exp; the combine kernel merges the splits.
+#include "kernels.h"
+
+namespace asd {
+namespace {
+
+constexpr int kRowsPerCta = 64;   // 4 warps x 16 query rows
+constexpr int kKeysPerTile = 64;
+constexpr int kAttnStages = 2;  // 2 CTAs per SM fit with D = 128
+
+// ---------------------------------------------------------------- mma helpers
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
+                                        uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr)
+               : "memory");
+}
+
+__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
+                                          uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr)
+               : "memory");
+}
+
+__device__ __forceinline__ void mma_bf16(float (&c)[4], const uint32_t (&a)[4], uint32_t b0,
+                                         uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
+      "{%8,%9}, {%0,%1,%2,%3};"
+      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+  __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&v);
+}
+
+// Tile layout in shared memory (the TMA 128-byte swizzle): [D/64 halves]
+// [64 rows][128 bytes]; 16-byte chunk c of row r sits at chunk c ^ (r & 7).
+__device__ __forceinline__ uint32_t sw_off(int row, int chunk) {
+  return static_cast<uint32_t>((chunk >> 3) * 8192 + row * 128 + (((chunk & 7) ^ (row & 7)) << 4));
+}
+
+__device__ __forceinline__ bool anc_bit(uint64_t lo, uint64_t hi, int j) {
+  return j < 64 ? ((lo >> j) & 1ull) : ((hi >> (j - 64)) & 1ull);
+}
+
+struct RowMap {
+  int s0, G, Hq, g, r0;
+  __device__ __forceinline__ size_t grow(int r) const {
+    const int rr = r0 + r;
+    const int i = rr / G;
+    return static_cast<size_t>(s0 + i) * Hq + g * G + (rr - i * G);
+  }
+};
+
+// ----------------------------------------------------------- bf16 tensor path
+template <int D>
+__global__ void __launch_bounds__(128) attn_bf16_kernel(const __grid_constant__ CUtensorMap tm_k,
+                                                        const __grid_constant__ CUtensorMap tm_v,
+                                                        const AttnParams p) {
+  constexpr int kTileBytes = kKeysPerTile * D * 2;
+  constexpr int kNH = D / 64;
+  constexpr int kChunks = D / 8;
+  extern __shared__ uint8_t smem_raw[];
+  __shared__ int s_abort;
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int rb = blockIdx.x, bg = blockIdx.y, z = blockIdx.z;
+  const int b = bg / p.Hkv, g = bg - b * p.Hkv;
+  if (p.seq_flags[b] & (kSeqBadTree | kSeqBadCtx)) return;
+  const int s0 = p.cu_nodes[b];
+  const int n = p.cu_nodes[b + 1] - s0;
+  const int R = n * p.G;
+  const int r0 = rb * kRowsPerCta;
+  if (r0 >= R) return;
+  const int nrows = min(kRowsPerCta, R - r0);
+  const bool is_tree = (z == p.n_splits);
+  int kbeg, kend;
+  if (is_tree) {
+    kbeg = 0;
+    kend = n;
+  } else {
+    kbeg = z * p.split_len;
+    kend = min(kbeg + p.split_len, p.ctx_len[b]);
+  }
+  const RowMap rm{s0, p.G, p.Hq, g, r0};
+  const size_t TH = static_cast<size_t>(p.T) * p.Hq;
+  if (kbeg >= kend) {
+    for (int r = tid; r < nrows; r += 128) p.part_lse[z * TH + rm.grow(r)] = -INFINITY;
+    return;
+  }
+
+  uint32_t base = smem_u32(smem_raw);
+  const uint32_t pad = (1024u - (base & 1023u)) & 1023u;
+  uint8_t* smem = smem_raw + pad;
+  base += pad;
+  const uint32_t sQ = base;
+  const uint32_t sK = sQ + kTileBytes;
+  const uint32_t sV = sK + kAttnStages * kTileBytes;
+  const uint32_t sBar = sV + kAttnStages * kTileBytes;
+  uint8_t* gQ = smem;
+  uint8_t* gK = smem + kTileBytes;
+  uint8_t* gV = gK + kAttnStages * kTileBytes;
+
+  // query rows -> shared memory (swizzled like the TMA tiles)
+  const __nv_bfloat16* q = static_cast<const __nv_bfloat16*>(p.q);
+  for (int c = tid; c < kRowsPerCta * kChunks; c += 128) {
+    const int r = c / kChunks, ch = c - r * kChunks;
+    uint4 v = make_uint4(0u, 0u, 0u, 0u);
+    if (r < nrows) v = *reinterpret_cast<const uint4*>(q + rm.grow(r) * D + ch * 8);
+    *reinterpret_cast<uint4*>(gQ + sw_off(r, ch)) = v;
+  }
+  if (tid == 0) {
+    s_abort = 0;
+    if (!is_tree) {
+      for (int s = 0; s < kAttnStages; ++s) mbar_init(sBar + 8 * s, 1);
+      fence_mbar_init();
+    }
+  }
+  __syncthreads();
+
+  const int ntiles = (kend - kbeg + kKeysPerTile - 1) / kKeysPerTile;
+  const int ps = p.page_size;
+  uint64_t pol = 0;
+
+  auto issue = [&](int t) {
+    const int stage = t % kAttnStages;
+    const int key0 = kbeg + t * kKeysPerTile;
+    const uint32_t dK = sK + stage * kTileBytes, dV = sV + stage * kTileBytes;
+    const uint32_t bar = sBar + 8 * stage;
+    if (ps == 0) {
+      const int row = (b * p.Hkv + g) * p.ctx_max + key0;
+      mbar_expect_tx(bar, 2 * kTileBytes);
+#pragma unroll
+      for (int h = 0; h < kNH; ++h) {
+        tma_load_2d(dK + h * 8192, &tm_k, bar, h * 64, row, pol);
+        tma_load_2d(dV + h * 8192, &tm_v, bar, h * 64, row, pol);
+      }
+    } else {
+      const int br = ps < 64 ? ps : 64;  // rows per box
+      const int nbox = kKeysPerTile / br;
+      int rows[kKeysPerTile / 8];  // at most 8 boxes (page_size >= 8)
+      int cnt = 0;
+      for (int j = 0; j < nbox; ++j) {
+        const int key = key0 + j * br;
+        rows[j] = -1;
+        if (key >= kend) continue;
+        const int page = p.page_table[static_cast<size_t>(b) * p.pages_per_seq + key / ps];
+        if (page < 0 || page >= p.num_pages) {
+          set_status(p.status, ASD_ERR_CTX_RANGE);
+          continue;
+        }
+        rows[j] = (page * p.Hkv + g) * ps + (key % ps);
+        ++cnt;
+      }
+      mbar_expect_tx(bar, static_cast<uint32_t>(cnt * 2 * kNH * br * 128));
+      for (int j = 0; j < nbox; ++j) {
+        if (rows[j] < 0) continue;
+#pragma unroll
+        for (int h = 0; h < kNH; ++h) {
+          tma_load_2d(dK + h * 8192 + j * br * 128, &tm_k, bar, h * 64, rows[j], pol);
+          tma_load_2d(dV + h * 8192 + j * br * 128, &tm_v, bar, h * 64, rows[j], pol);
+        }
+      }
+    }
+  };
+
+  if (!is_tree && tid == 0) {
+    pol = l2_policy_evict_first();
+    prefetch_tmap(&tm_k);
+    prefetch_tmap(&tm_v);
+    for (int t = 0; t < ntiles && t < kAttnStages; ++t) issue(t);
+  }
+
+  // Q fragments stay in registers for the whole kernel
+  uint32_t qa[D / 16][4];
+#pragma unroll
+  for (int ks = 0; ks < D / 16; ++ks) {
+    const int row = warp * 16 + (lane & 7) + (((lane >> 3) & 1) << 3);
+    const int chunk = 2 * ks + (lane >> 4);
+    ldsm_x4(sQ + sw_off(row, chunk), qa[ks][0], qa[ks][1], qa[ks][2], qa[ks][3]);
+  }
+
+  // ancestor masks of this thread's two rows (tree split)
+  const int rowA = warp * 16 + (lane >> 2), rowB = rowA + 8;
+  uint64_t aAlo = 0, aAhi = 0, aBlo = 0, aBhi = 0;
+  if (is_tree) {
+    if (rowA < nrows) {
+      const int node = s0 + (r0 + rowA) / p.G;
+      aAlo = p.anc[2 * node];
+      aAhi = p.anc[2 * node + 1];
+    }
+    if (rowB < nrows) {
+      const int node = s0 + (r0 + rowB) / p.G;
+      aBlo = p.anc[2 * node];
+      aBhi = p.anc[2 * node + 1];
+    }
+  }
+
+  float mA = -INFINITY, mB = -INFINITY, lA = 0.f, lB = 0.f;
+  float o[D / 8][4];
+#pragma unroll
+  for (int j = 0; j < D / 8; ++j) o[j][0] = o[j][1] = o[j][2] = o[j][3] = 0.f;
+  const float c = p.scale_log2;
+  const int kq = lane & 3;
+  const __nv_bfloat16* tk = static_cast<const __nv_bfloat16*>(p.tree_k);
+  const __nv_bfloat16* tv = static_cast<const __nv_bfloat16*>(p.tree_v);
+
+  for (int t = 0; t < ntiles; ++t) {
+    const int stage = t % kAttnStages;
+    const int key0 = kbeg + t * kKeysPerTile;
+    const int valid = min(kKeysPerTile, kend - key0);
+    uint8_t* gKs = gK + stage * kTileBytes;
+    uint8_t* gVs = gV + stage * kTileBytes;
+    if (is_tree) {
+      for (int cidx = tid; cidx < kKeysPerTile * kChunks; cidx += 128) {
+        const int r = cidx / kChunks, ch = cidx - r * kChunks;
+        uint4 kv = make_uint4(0u, 0u, 0u, 0u), vv = kv;
+        if (r < valid) {
+          const size_t off = (static_cast<size_t>(s0 + key0 + r) * p.Hkv + g) * D + ch * 8;
+          kv = *reinterpret_cast<const uint4*>(tk + off);
+          vv = *reinterpret_cast<const uint4*>(tv + off);
+        }
+        *reinterpret_cast<uint4*>(gKs + sw_off(r, ch)) = kv;
+        *reinterpret_cast<uint4*>(gVs + sw_off(r, ch)) = vv;
+      }
+    } else {
+      const bool ok = mbar_wait(sBar + 8 * stage, (t / kAttnStages) & 1);
+      if (!ok) {
+        set_status(p.status, ASD_ERR_TIMEOUT);
+        s_abort = 1;
+      } else if (valid < kKeysPerTile) {
+        // rows past the context may hold anything: zero V so that 0 * V stays 0
+        for (int cidx = tid; cidx < (kKeysPerTile - valid) * kChunks; cidx += 128) {
+          const int r = valid + cidx / kChunks, ch = cidx % kChunks;
+          *reinterpret_cast<uint4*>(gVs + sw_off(r, ch)) = make_uint4(0u, 0u, 0u, 0u);
+        }
+      }
+    }
+    __syncthreads();
+    if (s_abort) break;
+
+    const uint32_t aK = sK + stage * kTileBytes, aV = sV + stage * kTileBytes;
+    float sc[8][4];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) sc[j][0] = sc[j][1] = sc[j][2] = sc[j][3] = 0.f;
+#pragma unroll
+    for (int ks = 0; ks < D / 16; ++ks) {
+#pragma unroll
+      for (int nj = 0; nj < 4; ++nj) {
+        uint32_t b0, b1, b2, b3;
+        const int key = 16 * nj + (lane & 7) + ((lane >> 4) << 3);
+        const int chunk = 2 * ks + ((lane >> 3) & 1);
+        ldsm_x4(aK + sw_off(key, chunk), b0, b1, b2, b3);
+        mma_bf16(sc[2 * nj], qa[ks], b0, b1);
+        mma_bf16(sc[2 * nj + 1], qa[ks], b2, b3);
+      }
+    }
+    // mask and online softmax (scores in raw units; exp2 with the folded scale)
+    float mxA = -INFINITY, mxB = -INFINITY;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+#pragma unroll
+      for (int e = 0; e < 2; ++e) {
+        const int local = 8 * j + 2 * kq + e;
+        bool vA, vB;
+        if (is_tree) {
+          const int key = key0 + local;
+          vA = key < kend && anc_bit(aAlo, aAhi, key);
+          vB = key < kend && anc_bit(aBlo, aBhi, key);
+        } else {
+          vA = vB = local < valid;
+        }
+        sc[j][e] = vA ? sc[j][e] : -INFINITY;
+        sc[j][2 + e] = vB ? sc[j][2 + e] : -INFINITY;
+        mxA = fmaxf(mxA, sc[j][e]);
+        mxB = fmaxf(mxB, sc[j][2 + e]);
+      }
+    }
+    mxA = fmaxf(mxA, __shfl_xor_sync(0xffffffffu, mxA, 1));
+    mxA = fmaxf(mxA, __shfl_xor_sync(0xffffffffu, mxA, 2));
+    mxB = fmaxf(mxB, __shfl_xor_sync(0xffffffffu, mxB, 1));
+    mxB = fmaxf(mxB, __shfl_xor_sync(0xffffffffu, mxB, 2));
+    const float mnA = fmaxf(mA, mxA), mnB = fmaxf(mB, mxB);
+    const float muA = (mnA == -INFINITY) ? 0.f : mnA;
+    const float muB = (mnB == -INFINITY) ? 0.f : mnB;
+    const float alA = exp2f((mA - muA) * c), alB = exp2f((mB - muB) * c);
+    mA = mnA;
+    mB = mnB;
+    lA *= alA;
+    lB *= alB;
+#pragma unroll
+    for (int j = 0; j < D / 8; ++j) {
+      o[j][0] *= alA;
+      o[j][1] *= alA;
+      o[j][2] *= alB;
+      o[j][3] *= alB;
+    }
+    const float nA = -muA * c, nB = -muB * c;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      sc[j][0] = exp2f(fmaf(sc[j][0], c, nA));
+      sc[j][1] = exp2f(fmaf(sc[j][1], c, nA));
+      sc[j][2] = exp2f(fmaf(sc[j][2], c, nB));
+      sc[j][3] = exp2f(fmaf(sc[j][3], c, nB));
+      lA += sc[j][0] + sc[j][1];
+      lB += sc[j][2] + sc[j][3];
+    }
+    // O += P V
+#pragma unroll
+    for (int kk = 0; kk < 4; ++kk) {
+      uint32_t pa[4];
+      pa[0] = pack_bf16(sc[2 * kk][0], sc[2 * kk][1]);
+      pa[1] = pack_bf16(sc[2 * kk][2], sc[2 * kk][3]);
+      pa[2] = pack_bf16(sc[2 * kk + 1][0], sc[2 * kk + 1][1]);
+      pa[3] = pack_bf16(sc[2 * kk + 1][2], sc[2 * kk + 1][3]);
+#pragma unroll
+      for (int dp = 0; dp < D / 16; ++dp) {
+        uint32_t b0, b1, b2, b3;
+        const int key = 16 * kk + (lane & 7) + (((lane >> 3) & 1) << 3);
+        const int chunk = 2 * dp + (lane >> 4);
+        ldsm_x4_t(aV + sw_off(key, chunk), b0, b1, b2, b3);
+        mma_bf16(o[2 * dp], pa, b0, b1);
+        mma_bf16(o[2 * dp + 1], pa, b2, b3);
+      }
+    }
+    __syncthreads();  // every warp is done with this stage
+    if (!is_tree && tid == 0 && t + kAttnStages < ntiles) {
+      fence_proxy_async();
+      issue(t + kAttnStages);
+    }
+  }
+  if (s_abort) return;
+
+  lA += __shfl_xor_sync(0xffffffffu, lA, 1);
+  lA += __shfl_xor_sync(0xffffffffu, lA, 2);
+  lB += __shfl_xor_sync(0xffffffffu, lB, 1);
+  lB += __shfl_xor_sync(0xffffffffu, lB, 2);
+  const float iA = lA > 0.f ? 1.f / lA : 0.f, iB = lB > 0.f ? 1.f / lB : 0.f;
+  if (rowA < nrows) {
+    const size_t gr = rm.grow(rowA);
+    float* dst = p.part_o + (z * TH + gr) * D;
+#pragma unroll
+    for (int j = 0; j < D / 8; ++j)
+      *reinterpret_cast<float2*>(dst + 8 * j + 2 * kq) = make_float2(o[j][0] * iA, o[j][1] * iA);
+    if (kq == 0) p.part_lse[z * TH + gr] = (mA == -INFINITY) ? -INFINITY : mA * c + log2f(lA);
+  }
+  if (rowB < nrows) {
+    const size_t gr = rm.grow(rowB);
+    float* dst = p.part_o + (z * TH + gr) * D;
+#pragma unroll
+    for (int j = 0; j < D / 8; ++j)
+      *reinterpret_cast<float2*>(dst + 8 * j + 2 * kq) = make_float2(o[j][2] * iB, o[j][3] * iB);
+    if (kq == 0) p.part_lse[z * TH + gr] = (mB == -INFINITY) ? -INFINITY : mB * c + log2f(lB);
+  }
+}
+
+// ----------------------------------------------------------- fp32 SIMT path
+// One warp per query row; lanes split the head dimension.  Exact fp32 math for
+// the fp32 workloads (no reduced-precision tensor path).
+template <int D>
+__global__ void __launch_bounds__(128) attn_f32_kernel(const AttnParams p) {
+  constexpr int kPer = D / 32;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int rb = blockIdx.x, bg = blockIdx.y, z = blockIdx.z;
+  const int b = bg / p.Hkv, g = bg - b * p.Hkv;
+  if (p.seq_flags[b] & (kSeqBadTree | kSeqBadCtx)) return;
+  const int s0 = p.cu_nodes[b];
+  const int n = p.cu_nodes[b + 1] - s0;
+  const int R = n * p.G;
+  const int r0 = rb * kRowsPerCta;
+  if (r0 >= R) return;
+  const int nrows = min(kRowsPerCta, R - r0);
+  const bool is_tree = (z == p.n_splits);
+  int kbeg, kend;
+  if (is_tree) {
+    kbeg = 0;
+    kend = n;
+  } else {
+    kbeg = z * p.split_len;
+    kend = min(kbeg + p.split_len, p.ctx_len[b]);
+  }
+  const RowMap rm{s0, p.G, p.Hq, g, r0};
+  const size_t TH = static_cast<size_t>(p.T) * p.Hq;
+  const float* qp = static_cast<const float*>(p.q);
+  const float* kc = static_cast<const float*>(p.k_cache);
+  const float* vc = static_cast<const float*>(p.v_cache);
+  const float* tk = static_cast<const float*>(p.tree_k);
+  const float* tv = static_cast<const float*>(p.tree_v);
+  const float c = p.scale_log2;
+  const int ps = p.page_size;
+
+  for (int r = warp; r < nrows; r += 4) {
+    const size_t gr = rm.grow(r);
+    if (kbeg >= kend) {
+      if (lane == 0) p.part_lse[z * TH + gr] = -INFINITY;
+      continue;
+    }
+    float qv[kPer], ov[kPer];
+#pragma unroll
+    for (int k = 0; k < kPer; ++k) {
+      qv[k] = qp[gr * D + lane + 32 * k];
+      ov[k] = 0.f;
+    }
+    uint64_t alo = 0, ahi = 0;
+    if (is_tree) {
+      const int node = s0 + (r0 + r) / p.G;
+      alo = p.anc[2 * node];
+      ahi = p.anc[2 * node + 1];
+    }
+    float m = -INFINITY, l = 0.f;
+    for (int key = kbeg; key < kend; ++key) {
+      const float* kr;
+      const float* vr;
+      if (is_tree) {
+        if (!anc_bit(alo, ahi, key)) continue;
+        const size_t off = (static_cast<size_t>(s0 + key) * p.Hkv + g) * D;
+        kr = tk + off;
+        vr = tv + off;
+      } else if (ps == 0) {
+        const size_t off = ((static_cast<size_t>(b) * p.Hkv + g) * p.ctx_max + key) * D;
+        kr = kc + off;
+        vr = vc + off;
+      } else {
+        const int page = p.page_table[static_cast<size_t>(b) * p.pages_per_seq + key / ps];
+        if (page < 0 || page >= p.num_pages) {
+          if (lane == 0) set_status(p.status, ASD_ERR_CTX_RANGE);
+          continue;
+        }
+        const size_t off = ((static_cast<size_t>(page) * p.Hkv + g) * ps + key % ps) * D;
+        kr = kc + off;
+        vr = vc + off;
+      }
+      float dot = 0.f;
+#pragma unroll
+      for (int k = 0; k < kPer; ++k) dot = fmaf(qv[k], kr[lane + 32 * k], dot);
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) dot += __shfl_xor_sync(0xffffffffu, dot, off);
+      const float mn = fmaxf(m, dot);
+      const float al = exp2f((m - mn) * c);
+      const float pe = exp2f((dot - mn) * c);
+      l = l * al + pe;
+#pragma unroll
+      for (int k = 0; k < kPer; ++k) ov[k] = fmaf(pe, vr[lane + 32 * k], ov[k] * al);
+      m = mn;
+    }
+    const float inv = l > 0.f ? 1.f / l : 0.f;
+    float* dst = p.part_o + (z * TH + gr) * D;
+#pragma unroll
+    for (int k = 0; k < kPer; ++k) dst[lane + 32 * k] = ov[k] * inv;
+    if (lane == 0) p.part_lse[z * TH + gr] = (m == -INFINITY) ? -INFINITY : m * c + log2f(l);
+  }
+}
+
+// -------------------------------------------------------------------- combine
+template <typename OutT, int D>
+__global__ void __launch_bounds__(128) attn_combine_kernel(const AttnParams p) {
+  constexpr int kPer = D / 32;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const size_t TH = static_cast<size_t>(p.T) * p.Hq;
+  const size_t row = static_cast<size_t>(blockIdx.x) * 4 + warp;
+  if (row >= TH) return;
+  float M = -INFINITY;
+  for (int zz = 0; zz < p.n_parts; ++zz) M = fmaxf(M, p.part_lse[zz * TH + row]);
+  float acc[kPer];
+#pragma unroll
+  for (int k = 0; k < kPer; ++k) acc[k] = 0.f;
+  float wsum = 0.f;
+  if (M != -INFINITY) {
+    for (int zz = 0; zz < p.n_parts; ++zz) {
+      const float lz = p.part_lse[zz * TH + row];
+      if (lz == -INFINITY) continue;
+      const float w = exp2f(lz - M);
+      wsum += w;
+      const float* src = p.part_o + (zz * TH + row) * D + lane * kPer;
+      if constexpr (kPer == 4) {
+        const float4 v = *reinterpret_cast<const float4*>(src);
+        acc[0] = fmaf(w, v.x, acc[0]);
+        acc[1] = fmaf(w, v.y, acc[1]);
+        acc[2] = fmaf(w, v.z, acc[2]);
+        acc[3] = fmaf(w, v.w, acc[3]);
+      } else {
+        const float2 v = *reinterpret_cast<const float2*>(src);
+        acc[0] = fmaf(w, v.x, acc[0]);
+        acc[1] = fmaf(w, v.y, acc[1]);
+      }
+    }
+  }
+  const float inv = wsum > 0.f ? 1.f / wsum : 0.f;
+  OutT* out = static_cast<OutT*>(p.out) + row * D + lane * kPer;
+#pragma unroll
+  for (int k = 0; k < kPer; ++k) out[k] = from_f32<OutT>(acc[k] * inv);
+}
+
+}  // namespace
+
+size_t attn_bf16_smem_bytes(int D) {
+  const size_t tile = static_cast<size_t>(kKeysPerTile) * D * 2;
+  return 1024 + tile * (1 + 2 * kAttnStages) + 8 * kAttnStages;
+}
+
+static dim3 attn_grid(const AttnParams& p) {
+  const int rblocks = (p.max_nodes * p.G + kRowsPerCta - 1) / kRowsPerCta;
+  return dim3(rblocks, p.B * p.Hkv, p.n_parts);
+}
+
+cudaError_t launch_attention_bf16(const AttnParams& p, const CUtensorMap& tm_k,
+                                  const CUtensorMap& tm_v, cudaStream_t s) {
+  const size_t smem = attn_bf16_smem_bytes(p.D);
+  cudaError_t err;
+  if (p.D == 128) {
+    err = cudaFuncSetAttribute(attn_bf16_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               static_cast<int>(smem));
+    if (err != cudaSuccess) return err;
+    attn_bf16_kernel<128><<<attn_grid(p), 128, smem, s>>>(tm_k, tm_v, p);
+  } else {
+    err = cudaFuncSetAttribute(attn_bf16_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               static_cast<int>(smem));
+    if (err != cudaSuccess) return err;
+    attn_bf16_kernel<64><<<attn_grid(p), 128, smem, s>>>(tm_k, tm_v, p);
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_attention_f32(const AttnParams& p, cudaStream_t s) {
+  if (p.D == 128)
+    attn_f32_kernel<128><<<attn_grid(p), 128, 0, s>>>(p);
+  else
+    attn_f32_kernel<64><<<attn_grid(p), 128, 0, s>>>(p);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_attention_combine(const AttnParams& p, bool bf16, cudaStream_t s) {
+  const size_t rows = static_cast<size_t>(p.T) * p.Hq;
+  const dim3 grid(static_cast<unsigned>((rows + 3) / 4));
+  if (bf16) {
+    if (p.D == 128) attn_combine_kernel<__nv_bfloat16, 128><<<grid, 128, 0, s>>>(p);
+    else attn_combine_kernel<__nv_bfloat16, 64><<<grid, 128, 0, s>>>(p);
+  } else {
+    if (p.D == 128) attn_combine_kernel<float, 128><<<grid, 128, 0, s>>>(p);
+    else attn_combine_kernel<float, 64><<<grid, 128, 0, s>>>(p);
+  }
+  return cudaGetLastError();
+}
+
+}  // namespace asd

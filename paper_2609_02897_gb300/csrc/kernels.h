@@ -1,0 +1,117 @@
+// Internal interface between the C-ABI layer (asd_api.cu) and the kernels.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "common.cuh"
+
+namespace asd {
+
+// ------------------------------------------------------------ tree preparation
+struct PrepParams {
+  const int32_t* parent;
+  const int32_t* tokens;    // may be null (attention-only call)
+  const int32_t* cu_nodes;
+  const int32_t* ctx_len;   // may be null
+  int* status;
+  int* seq_flags;
+  uint64_t* anc;
+  int32_t* child_start;
+  int32_t* child_cnt;
+  int32_t* child_tok;
+  int32_t* child_id;
+  float* l_draft;           // may be null; set to NaN
+  int B, T, vocab, max_nodes, ctx_max;
+};
+cudaError_t launch_tree_prep(const PrepParams& p, cudaStream_t s);
+
+// ------------------------------------------------------------------ attention
+struct AttnParams {
+  const void* q;            // [T, Hq, D]
+  const void* k_cache;      // contiguous [B,Hkv,ctx_max,D] / paged [P,Hkv,ps,D]
+  const void* v_cache;
+  const void* tree_k;       // [T, Hkv, D]
+  const void* tree_v;
+  const int32_t* cu_nodes;
+  const int32_t* ctx_len;
+  const int32_t* page_table;  // [B, ctx_max / ps] or null
+  const int* seq_flags;
+  const uint64_t* anc;
+  float* part_o;            // [n_parts][T*Hq][D]
+  float* part_lse;          // [n_parts][T*Hq]
+  int* status;
+  void* out;                // [T, Hq, D]
+  int B, T, Hq, Hkv, G, D;
+  int ctx_max, page_size, pages_per_seq, num_pages;
+  int n_splits, split_len, n_parts, max_nodes;
+  float scale_log2;         // log2(e) / sqrt(D)
+};
+// bf16 path: tensor-core (mma.sync) split-KV kernel fed by TMA; tm_k / tm_v are
+// 2D tensor maps over the context cache rows (box 64 x min(64, rows per page)).
+cudaError_t launch_attention_bf16(const AttnParams& p, const CUtensorMap& tm_k,
+                                  const CUtensorMap& tm_v, cudaStream_t s);
+cudaError_t launch_attention_f32(const AttnParams& p, cudaStream_t s);
+cudaError_t launch_attention_combine(const AttnParams& p, bool bf16, cudaStream_t s);
+
+// -------------------------------------------------------------------- LM head
+struct LmParams {
+  const void* hidden;       // [T, K]
+  const void* w;            // [V, K]
+  const int32_t* child_start;
+  const int32_t* child_cnt;
+  const int32_t* child_tok;
+  const int32_t* child_id;
+  LmPartial* part;          // [T][g_lm]
+  float* l_draft;           // [T]
+  int* status;
+  int T, K, V, g_lm;
+};
+constexpr int kLmStages = 4;
+constexpr int kLmTileN = 256;      // vocabulary rows per MMA tile
+constexpr int kLmBoxRows = 32;     // vocabulary rows per TMA box
+size_t lmhead_tc_smem_bytes();
+// bf16 path: tcgen05/TMEM GEMM with the fused max/argmax/sum-exp/l_draft epilogue.
+cudaError_t launch_lmhead_bf16(const LmParams& p, const CUtensorMap& tm_hidden,
+                               const CUtensorMap& tm_w, cudaStream_t s);
+cudaError_t launch_lmhead_f32(const LmParams& p, cudaStream_t s);
+
+// --------------------------------------- finalize / accepted path / K/V commit
+enum TailMode : int { kTailFinalize = 1, kTailWalk = 2, kTailCompact = 4 };
+struct TailParams {
+  int mode;
+  const int32_t* parent;
+  const int32_t* tokens;
+  const int32_t* cu_nodes;
+  const int* seq_flags;       // from tree preparation, or null
+  // finalize
+  const LmPartial* part;
+  int g_lm;
+  float ln_tau;
+  float* row_max;
+  int32_t* row_argmax;        // written by finalize, read by walk
+  float* row_lse;
+  const float* l_draft;
+  float* ratio;
+  uint8_t* accept;            // written by finalize, read by walk
+  // walk
+  int32_t* path;              // [B, max_path]
+  int32_t* path_len;
+  int32_t* bonus;
+  int32_t* n_promoted;
+  // compact
+  const void* tree_k;
+  const void* tree_v;
+  void* k_cache;
+  void* v_cache;
+  const int32_t* ctx_len;
+  const int32_t* page_table;
+  int32_t* ctx_len_out;
+  int* status;
+  int B, T, Hkv, D, elem_bytes, max_nodes, max_path;
+  int ctx_max, page_size, pages_per_seq, num_pages;
+};
+cudaError_t launch_tail(const TailParams& p, cudaStream_t s);
+
+}  // namespace asd

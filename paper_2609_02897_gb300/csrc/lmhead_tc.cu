@@ -1,0 +1,320 @@
+// LM head of the verify pass fused with the margin-rule statistics (Eq. 1),
+// bf16 inputs on the sm_103a tensor cores (tcgen05, accumulators in TMEM).
+//
+// logits[node, v] = hidden[node, :] . W[v, :] are computed as
+//   D[128 nodes, up to 256 vocab rows] = hidden_tile[128, K] x W_tile[N, K]^T
+// so that TMEM lane i holds node row i and the epilogue thread that owns lane
+// i reduces its row over the vocabulary without any cross-thread exchange:
+// running max, lowest argmax, sum of exp and the drafted tokens' logits.
+// Logits never leave the SM.  Each CTA owns one contiguous vocabulary range
+// (one CTA per SM, ranges balanced to 32 rows), streams its slice of W once
+// per 128-node tile through a 4-stage TMA ring, and writes one partial
+// (max, argmax, sum-exp) per node; the tail kernel merges the ranges.
+//
+// Warp roles (192 threads): warp 0 TMA producer, warp 1 TMEM allocator and
+// MMA issuer, warps 2-5 epilogue (TMEM lane quarters 2, 3, 0, 1).
+#include "kernels.h"
+#include "lm_epilogue.cuh"
+
+namespace asd {
+namespace {
+
+constexpr int kM = 128;                        // node rows per MMA = TMEM lanes
+constexpr int kKB = 64;                        // hidden elements per k-block (128 B)
+constexpr int kATile = kM * 128;               // 16 KB
+constexpr int kBTile = kLmTileN * 128;         // 32 KB
+constexpr int kStage = kATile + kBTile;
+constexpr int kBoxBytes = kLmBoxRows * 128;    // 4 KB
+constexpr uint32_t kTmemCols = 2 * kLmTileN;   // two accumulators
+
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
+  uint64_t d = static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);  // start address >> 4
+  d |= static_cast<uint64_t>(1) << 16;                          // leading offset (unused, SW128 K-major)
+  d |= static_cast<uint64_t>(1024 >> 4) << 32;                  // stride: 8 rows x 128 B
+  d |= static_cast<uint64_t>(1) << 46;                          // tcgen05 descriptor version
+  d |= static_cast<uint64_t>(2) << 61;                          // 128-byte swizzle
+  return d;
+}
+
+// kind::f16 instruction descriptor: D f32, A/B bf16, both K-major, M x N.
+__device__ __forceinline__ uint32_t idesc_bf16(int m, int n) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | (static_cast<uint32_t>(n >> 3) << 17) |
+         (static_cast<uint32_t>(m >> 4) << 24);
+}
+
+__device__ __forceinline__ void tmem_alloc(uint32_t dst_smem, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst_smem),
+               "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void tmem_relinquish() {
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_mma(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
+                                       uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+__device__ __forceinline__ void tc_commit(uint32_t bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+      : "memory");
+}
+
+// 32 consecutive TMEM columns of this warp's 32 lanes -> v[0..31] (one lane each).
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, "
+      "%12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, "
+      "%30, %31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]),
+        "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]),
+        "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+  // the wait names every destination register so no use can move above it
+  asm volatile("tcgen05.wait::ld.sync.aligned;"
+               : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]),
+                 "+r"(r[6]), "+r"(r[7]), "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]),
+                 "+r"(r[12]), "+r"(r[13]), "+r"(r[14]), "+r"(r[15]), "+r"(r[16]), "+r"(r[17]),
+                 "+r"(r[18]), "+r"(r[19]), "+r"(r[20]), "+r"(r[21]), "+r"(r[22]), "+r"(r[23]),
+                 "+r"(r[24]), "+r"(r[25]), "+r"(r[26]), "+r"(r[27]), "+r"(r[28]), "+r"(r[29]),
+                 "+r"(r[30]), "+r"(r[31])
+               :
+               : "memory");
+#pragma unroll
+  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+__global__ void __launch_bounds__(192, 1)
+    lmhead_tc_kernel(const __grid_constant__ CUtensorMap tm_h,
+                     const __grid_constant__ CUtensorMap tm_w, const LmParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  __shared__ __align__(8) uint64_t s_full[kLmStages];
+  __shared__ __align__(8) uint64_t s_empty[kLmStages];
+  __shared__ __align__(8) uint64_t s_tfull[2];
+  __shared__ __align__(8) uint64_t s_tempty[2];
+  __shared__ uint32_t s_tmem;
+  __shared__ volatile int s_abort;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  // this CTA's vocabulary range, in whole groups of kLmBoxRows rows
+  const int ngroups = (p.V + kLmBoxRows - 1) / kLmBoxRows;
+  const int gs = static_cast<int>(static_cast<long long>(blockIdx.x) * ngroups / p.g_lm);
+  const int ge = static_cast<int>(static_cast<long long>(blockIdx.x + 1) * ngroups / p.g_lm);
+  const int vs = gs * kLmBoxRows;
+  const int ve = min(p.V, ge * kLmBoxRows);
+  const int nvt = ve > vs ? (ve - vs + kLmTileN - 1) / kLmTileN : 0;
+  const int nnt = (p.T + kM - 1) / kM;
+  const int nkb = (p.K + kKB - 1) / kKB;
+
+  uint32_t base = smem_u32(smem_raw);
+  base += (1024u - (base & 1023u)) & 1023u;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kLmStages; ++s) {
+      mbar_init(smem_u32(&s_full[s]), 1);
+      mbar_init(smem_u32(&s_empty[s]), 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(smem_u32(&s_tfull[a]), 1);
+      mbar_init(smem_u32(&s_tempty[a]), 4);
+    }
+    s_abort = 0;
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(&s_tmem), kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = s_tmem;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ TMA producer
+    uint64_t pol_w = 0, pol_h = 0;
+    if (lane == 0) {
+      prefetch_tmap(&tm_h);
+      prefetch_tmap(&tm_w);
+      pol_w = l2_policy_evict_first();
+      pol_h = l2_policy_evict_last();
+    }
+    int stage = 0;
+    uint32_t ph = 0;
+    bool ok = true;
+    for (int nt = 0; nt < nnt && ok; ++nt) {
+      for (int vt = 0; vt < nvt && ok; ++vt) {
+        const int v0 = vs + vt * kLmTileN;
+        const int nbox = (min(kLmTileN, ve - v0) + kLmBoxRows - 1) / kLmBoxRows;
+        for (int kb = 0; kb < nkb; ++kb) {
+          const uint32_t full = smem_u32(&s_full[stage]);
+          ok = __shfl_sync(0xffffffffu, mbar_wait(smem_u32(&s_empty[stage]), ph ^ 1u), 0);
+          if (!ok || s_abort) {
+            ok = false;
+            break;
+          }
+          if (lane == 0) {
+            const uint32_t a_s = base + stage * kStage;
+            const uint32_t b_s = a_s + kATile;
+            mbar_expect_tx(full, static_cast<uint32_t>(kATile + nbox * kBoxBytes));
+            tma_load_2d(a_s, &tm_h, full, kb * kKB, nt * kM, pol_h);
+            for (int j = 0; j < nbox; ++j)
+              tma_load_2d(b_s + j * kBoxBytes, &tm_w, full, kb * kKB, v0 + j * kLmBoxRows, pol_w);
+          }
+          __syncwarp();
+          if (++stage == kLmStages) {
+            stage = 0;
+            ph ^= 1u;
+          }
+        }
+      }
+    }
+    if (!ok && lane == 0) {
+      set_status(p.status, ASD_ERR_TIMEOUT);
+      s_abort = 1;
+    }
+  } else if (warp == 1) {
+    // --------------------------------------------------------------- MMA issuer
+    int stage = 0;
+    uint32_t ph = 0;
+    int acc = 0;
+    uint32_t aph = 0;
+    bool ok = true;
+    for (int nt = 0; nt < nnt && ok; ++nt) {
+      for (int vt = 0; vt < nvt && ok; ++vt) {
+        const int v0 = vs + vt * kLmTileN;
+        const int nrows = min(kLmTileN, ve - v0);
+        const uint32_t idesc = idesc_bf16(kM, (nrows + 15) & ~15);
+        ok = __shfl_sync(0xffffffffu, mbar_wait(smem_u32(&s_tempty[acc]), aph ^ 1u), 0);
+        if (!ok || s_abort) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d = tmem + static_cast<uint32_t>(acc * kLmTileN);
+        for (int kb = 0; kb < nkb; ++kb) {
+          ok = __shfl_sync(0xffffffffu, mbar_wait(smem_u32(&s_full[stage]), ph), 0);
+          if (!ok || s_abort) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          if (lane == 0) {
+            const uint32_t a_s = base + stage * kStage;
+            const uint32_t b_s = a_s + kATile;
+#pragma unroll
+            for (int k = 0; k < kKB / 16; ++k)
+              tc_mma(d, sw128_desc(a_s + 32 * k), sw128_desc(b_s + 32 * k), idesc,
+                     (kb | k) != 0 ? 1u : 0u);
+            tc_commit(smem_u32(&s_empty[stage]));
+          }
+          __syncwarp();
+          if (++stage == kLmStages) {
+            stage = 0;
+            ph ^= 1u;
+          }
+        }
+        if (!ok) break;
+        if (lane == 0) tc_commit(smem_u32(&s_tfull[acc]));
+        __syncwarp();
+        acc ^= 1;
+        if (acc == 0) aph ^= 1u;
+      }
+    }
+    if (!ok && lane == 0) {
+      set_status(p.status, ASD_ERR_TIMEOUT);
+      s_abort = 1;
+    }
+  } else {
+    // ----------------------------------------------------------------- epilogue
+    const int q = warp & 3;
+    const int row = q * 32 + lane;
+    int acc = 0;
+    uint32_t aph = 0;
+    bool ok = true;
+    for (int nt = 0; nt < nnt && ok; ++nt) {
+      const int node = nt * kM + row;
+      const bool active = node < p.T;
+      RowState st;
+      row_state_init(st, active, node, vs, p.child_start, p.child_cnt, p.child_tok, p.T);
+      for (int vt = 0; vt < nvt; ++vt) {
+        const int v0 = vs + vt * kLmTileN;
+        const int nrows = min(kLmTileN, ve - v0);
+        ok = __shfl_sync(0xffffffffu, mbar_wait(smem_u32(&s_tfull[acc]), aph), 0);
+        if (!ok || s_abort) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t taddr = tmem + (static_cast<uint32_t>(q * 32) << 16) +
+                               static_cast<uint32_t>(acc * kLmTileN);
+        const int nchunks = (nrows + 31) / 32;
+        for (int c = 0; c < nchunks; ++c) {
+          float r[32];
+          tmem_ld32(taddr + 32 * c, r);
+          if (active)
+            row_chunk(st, r, v0 + 32 * c, min(32, nrows - 32 * c), p.child_tok, p.child_id,
+                      p.l_draft, p.T);
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(smem_u32(&s_tempty[acc]));
+        acc ^= 1;
+        if (acc == 0) aph ^= 1u;
+      }
+      if (ok && active) {
+        LmPartial part;
+        part.m = st.m;
+        part.s = st.s;
+        part.a = st.a;
+        part.pad = 0;
+        p.part[static_cast<size_t>(node) * p.g_lm + blockIdx.x] = part;
+      }
+    }
+    if (!ok && lane == 0) {
+      set_status(p.status, ASD_ERR_TIMEOUT);
+      s_abort = 1;
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc(tmem, kTmemCols);
+}
+
+}  // namespace
+
+size_t lmhead_tc_smem_bytes() { return 1024 + static_cast<size_t>(kLmStages) * kStage; }
+
+cudaError_t launch_lmhead_bf16(const LmParams& p, const CUtensorMap& tm_hidden,
+                               const CUtensorMap& tm_w, cudaStream_t s) {
+  const size_t smem = lmhead_tc_smem_bytes();
+  cudaError_t err = cudaFuncSetAttribute(lmhead_tc_kernel,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(smem));
+  if (err != cudaSuccess) return err;
+  lmhead_tc_kernel<<<p.g_lm, 192, smem, s>>>(tm_hidden, tm_w, p);
+  return cudaGetLastError();
+}
+
+}  // namespace asd

@@ -1,0 +1,257 @@
+// Per-sequence tail of the verify step, one CTA of 128 threads per sequence
+// (thread i owns local node i).  Three stages, selected by TailParams::mode:
+//  finalize  merge the LM head's per-range partials of every row into
+//            row_max / row_argmax / row_lse and evaluate the margin rule for
+//            every drafted node: ratio = exp(l_draft - row_max[parent]) (Eq. 1),
+//            accept = strict match of the parent row's top-1 or ratio >= tau
+//            (compared as l_draft - row_max >= ln tau);
+//  walk      choose the longest root-to-node path of accepted nodes, ties to the
+//            lexicographically smallest node sequence (Sec. 3.2): heights of
+//            accepted subtrees bottom-up by depth, then from the root follow
+//            the lowest-index accepted child whose height is one less;
+//  compact   copy the path's tree K/V into cache slots ctx_len .. ctx_len +
+//            path_len - 1 (contiguous or through the page table).
+#include <climits>
+
+#include "kernels.h"
+
+namespace asd {
+namespace {
+
+__device__ __forceinline__ void merge_part(float& m, float& s, int& a, float m2, float s2,
+                                           int a2) {
+  if (m2 == -INFINITY) return;
+  if (m == -INFINITY) {
+    m = m2;
+    s = s2;
+    a = a2;
+    return;
+  }
+  const float M = fmaxf(m, m2);
+  s = s * exp2f((m - M) * kLog2e) + s2 * exp2f((m2 - M) * kLog2e);
+  if (m2 > m) a = a2;
+  else if (m2 == m) a = min(a, a2);
+  m = M;
+}
+
+__global__ void __launch_bounds__(kMaxNodes) tail_kernel(const TailParams p) {
+  __shared__ int s_par[kMaxNodes];
+  __shared__ int s_tok[kMaxNodes];
+  __shared__ int s_arg[kMaxNodes];
+  __shared__ float s_max[kMaxNodes];
+  __shared__ int s_acc[kMaxNodes];
+  __shared__ int s_dep[kMaxNodes];
+  __shared__ int s_h[kMaxNodes];
+  __shared__ int s_bc[kMaxNodes];
+  __shared__ int s_path[kMaxNodes];
+  __shared__ int s_maxd, s_len, s_skip;
+
+  const int b = blockIdx.x;
+  const int i = threadIdx.x;
+  const int warp = i >> 5, lane = i & 31;
+  const int s = p.cu_nodes[b];
+  const int e = p.cu_nodes[b + 1];
+  const bool seq_ok = (s >= 0) && (e > s) && (e <= p.T) && (e - s <= p.max_nodes);
+  if (!seq_ok) {
+    if (i == 0) {
+      set_status(p.status, ASD_ERR_TREE);
+      if (p.mode & kTailWalk) {
+        p.path_len[b] = 0;
+        p.bonus[b] = -1;
+        p.n_promoted[b] = 0;
+      }
+      if ((p.mode & kTailCompact) && p.ctx_len_out) p.ctx_len_out[b] = p.ctx_len[b];
+    }
+    return;
+  }
+  const int n = e - s;
+
+  bool okn = true;
+  if (i < n) {
+    // the standalone commit has no parent array: it only needs the path
+    const int par = p.parent ? p.parent[s + i] : (i == 0 ? -1 : 0);
+    okn = (i == 0) ? (par == -1) : (par >= 0 && par < i);
+    s_par[i] = okn ? par : -1;
+    s_tok[i] = p.tokens ? p.tokens[s + i] : 0;
+  }
+  const int tree_bad = __syncthreads_or(!okn);
+  const int flags = p.seq_flags ? p.seq_flags[b] : 0;
+  if (i == 0) {
+    if (tree_bad) set_status(p.status, ASD_ERR_TREE);
+    s_skip = (tree_bad || flags) ? 1 : 0;
+    s_maxd = 0;
+    s_len = 0;
+  }
+
+  // ---------------------------------------------------------------- finalize
+  if (p.mode & kTailFinalize) {
+    if (!tree_bad) {
+      for (int r = warp; r < n; r += 4) {
+        const size_t node = static_cast<size_t>(s + r);
+        float m = -INFINITY, sm = 0.f;
+        int a = INT_MAX;
+        for (int g = lane; g < p.g_lm; g += 32) {
+          const LmPartial q = p.part[node * p.g_lm + g];
+          merge_part(m, sm, a, q.m, q.s, q.a);
+        }
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) {
+          const float m2 = __shfl_xor_sync(0xffffffffu, m, off);
+          const float s2 = __shfl_xor_sync(0xffffffffu, sm, off);
+          const int a2 = __shfl_xor_sync(0xffffffffu, a, off);
+          merge_part(m, sm, a, m2, s2, a2);
+        }
+        if (lane == 0) {
+          p.row_max[node] = m;
+          p.row_argmax[node] = a;
+          p.row_lse[node] = m + logf(sm);
+          s_max[r] = m;
+          s_arg[r] = a;
+        }
+      }
+    }
+    __syncthreads();
+    if (i < n && !tree_bad) {
+      int acc = 1;
+      float ratio = __int_as_float(0x7fc00000);
+      if (i > 0) {
+        const int pp = s_par[i];
+        const float d = p.l_draft[s + i] - s_max[pp];
+        const bool strict = s_tok[i] == s_arg[pp];
+        ratio = expf(d);
+        acc = (strict || d >= p.ln_tau) ? 1 : 0;
+      }
+      p.ratio[s + i] = ratio;
+      p.accept[s + i] = static_cast<uint8_t>(acc);
+      s_acc[i] = acc;
+    }
+  } else if (p.mode & kTailWalk) {
+    if (i < n) {
+      s_acc[i] = p.accept[s + i] != 0 ? 1 : 0;
+      s_arg[i] = p.row_argmax[s + i];
+    }
+  }
+  __syncthreads();
+
+  // -------------------------------------------------------------------- walk
+  if (p.mode & kTailWalk) {
+    if (!s_skip) {
+      if (i < n) {
+        int d = 0, u = i;
+        while (s_par[u] >= 0) {
+          u = s_par[u];
+          ++d;
+        }
+        s_dep[i] = d;
+        s_h[i] = 1;
+        s_bc[i] = INT_MAX;
+        atomicMax(&s_maxd, d);
+      }
+      __syncthreads();
+      for (int dd = s_maxd; dd >= 1; --dd) {
+        if (i < n && s_dep[i] == dd && s_acc[i]) atomicMax(&s_h[s_par[i]], s_h[i] + 1);
+        __syncthreads();
+      }
+      if (i > 0 && i < n && s_acc[i] && s_h[i] == s_h[s_par[i]] - 1) atomicMin(&s_bc[s_par[i]], i);
+      __syncthreads();
+      if (i == 0) {
+        int u = 0, len = 0, promoted = 0;
+        s_path[len++] = 0;
+        while (s_bc[u] != INT_MAX && len < kMaxNodes) {
+          const int c = s_bc[u];
+          if (s_tok[c] != s_arg[u]) ++promoted;
+          s_path[len++] = c;
+          u = c;
+        }
+        if (len > p.max_path) {
+          set_status(p.status, ASD_ERR_SHAPE);
+          len = 0;
+        }
+        s_len = len;
+        p.path_len[b] = len;
+        p.bonus[b] = len > 0 ? s_arg[u] : -1;
+        p.n_promoted[b] = len > 0 ? promoted : 0;
+      }
+      __syncthreads();
+      for (int k = i; k < p.max_path; k += kMaxNodes)
+        p.path[static_cast<size_t>(b) * p.max_path + k] = k < s_len ? s_path[k] : -1;
+    } else {
+      for (int k = i; k < p.max_path; k += kMaxNodes)
+        p.path[static_cast<size_t>(b) * p.max_path + k] = -1;
+      if (i == 0) {
+        p.path_len[b] = 0;
+        p.bonus[b] = -1;
+        p.n_promoted[b] = 0;
+      }
+    }
+  } else if (p.mode & kTailCompact) {
+    // standalone commit: the path comes from the caller
+    if (i == 0) {
+      int len = p.path_len[b];
+      bool ok = !s_skip && len >= 0 && len <= p.max_path && len <= n;
+      for (int k = 0; ok && k < len; ++k) {
+        const int u = p.path[static_cast<size_t>(b) * p.max_path + k];
+        if (u < 0 || u >= n) ok = false;
+        else s_path[k] = u;
+      }
+      if (!ok) {
+        set_status(p.status, ASD_ERR_SHAPE);
+        len = 0;
+        s_skip = 1;
+      }
+      s_len = len;
+    }
+  }
+  __syncthreads();
+
+  // ------------------------------------------------------------------ commit
+  if (p.mode & kTailCompact) {
+    const int ctx = p.ctx_len[b];
+    const int len = s_len;
+    const bool ctx_ok = ctx >= 0 && ctx + len <= p.ctx_max;
+    if (i == 0 && !ctx_ok && !s_skip) set_status(p.status, ASD_ERR_CTX_RANGE);
+    if (s_skip || !ctx_ok) {
+      if (i == 0) p.ctx_len_out[b] = ctx;
+      return;
+    }
+    const int row_bytes = p.D * p.elem_bytes;
+    const int chunks = row_bytes / 16;
+    const int per_node = p.Hkv * chunks;
+    const uint8_t* tk = static_cast<const uint8_t*>(p.tree_k);
+    const uint8_t* tv = static_cast<const uint8_t*>(p.tree_v);
+    uint8_t* kc = static_cast<uint8_t*>(p.k_cache);
+    uint8_t* vc = static_cast<uint8_t*>(p.v_cache);
+    for (int idx = i; idx < len * per_node; idx += kMaxNodes) {
+      const int k = idx / per_node;
+      const int rem = idx - k * per_node;
+      const int g = rem / chunks;
+      const int ch = rem - g * chunks;
+      const size_t src = (static_cast<size_t>(s + s_path[k]) * p.Hkv + g) * row_bytes + ch * 16;
+      const int slot = ctx + k;
+      size_t dst;
+      if (p.page_size == 0) {
+        dst = ((static_cast<size_t>(b) * p.Hkv + g) * p.ctx_max + slot) * row_bytes + ch * 16;
+      } else {
+        const int page = p.page_table[static_cast<size_t>(b) * p.pages_per_seq + slot / p.page_size];
+        if (page < 0 || page >= p.num_pages) {
+          set_status(p.status, ASD_ERR_CTX_RANGE);
+          continue;
+        }
+        dst = ((static_cast<size_t>(page) * p.Hkv + g) * p.page_size + slot % p.page_size) *
+                  row_bytes + ch * 16;
+      }
+      *reinterpret_cast<uint4*>(kc + dst) = *reinterpret_cast<const uint4*>(tk + src);
+      *reinterpret_cast<uint4*>(vc + dst) = *reinterpret_cast<const uint4*>(tv + src);
+    }
+    if (i == 0) p.ctx_len_out[b] = ctx + len;
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_tail(const TailParams& p, cudaStream_t s) {
+  tail_kernel<<<p.B, kMaxNodes, 0, s>>>(p);
+  return cudaGetLastError();
+}
+
+}  // namespace asd

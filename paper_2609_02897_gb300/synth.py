@@ -245,22 +245,25 @@ class Workload:
         return np.unique(gp[gp >= 0])
 
 
-def _spec(config: int, small: bool) -> dict:
+def _spec(config: int, small: bool, overrides: Optional[dict] = None) -> dict:
     s = dict(WORKLOADS[config])
     if small:
         s.update(SMALL[config])
+    if overrides:
+        s.update(overrides)
     return s
 
 
 def make_workload(config: int, rep: int = 0, small: bool = False,
-                  tree_override: Optional[list] = None) -> Workload:
+                  tree_override: Optional[list] = None,
+                  overrides: Optional[dict] = None) -> Workload:
     """Draw every input of one verify step except the drafted tokens.
 
     Seeds: numpy PCG64 with seed 1000*config + rep (+ 500 for the reduced
     variant).  Weights ~ N(0, 0.02); hidden states, queries, keys and values
     ~ N(0, 1).
     """
-    s = _spec(config, small)
+    s = _spec(config, small, overrides)
     seed = 1000 * config + rep + (500 if small else 0)
     rng = np.random.Generator(np.random.PCG64(seed))
     bf16 = s["dtype"] == "bf16"
@@ -272,7 +275,7 @@ def make_workload(config: int, rep: int = 0, small: bool = False,
     for b in range(B):
         t = s["tree"]
         if tree_override is not None:
-            par = np.asarray(tree_override[b], dtype=np.int32)
+            par = np.asarray(tree_override[b % len(tree_override)], dtype=np.int32)
         elif t == "c1":
             par = tree_fixed_c1()
         elif t[0] == "eagle":
