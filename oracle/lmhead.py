@@ -41,9 +41,12 @@ def topk_tokens(hidden, W, rows, k=5):
     (equal logits ordered by token id)."""
     lg = logits_rows(hidden, W, rows)
     out = np.empty((len(rows), k), dtype=np.int64)
+    kk = min(k, lg.shape[1])
     for r in range(len(rows)):
-        order = np.lexsort((np.arange(lg.shape[1]), -lg[r]))
-        out[r] = order[:k]
+        kth = np.partition(lg[r], lg.shape[1] - kk)[lg.shape[1] - kk]
+        cand = np.nonzero(lg[r] >= kth)[0]          # every id tied with the k-th value too
+        order = cand[np.lexsort((cand, -lg[r, cand]))]
+        out[r, :kk] = order[:kk]
     return out
 
 
