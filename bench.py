@@ -246,6 +246,7 @@ def run_asd(args):
 
     wl = synth.make_workload(CONFIG, rep=rank)
     synth.attach_tokens(wl, ranks_torch(wl, device))
+    torch.cuda.empty_cache()
     bf = torch.bfloat16
 
     def f(x):
