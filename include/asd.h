@@ -223,6 +223,38 @@ asd_status asd_get_device_status(const void* workspace, int32_t* status_out, voi
 const char* asd_status_string(int32_t status);
 int32_t asd_abi_version(void);
 
+/*
+ * Allocation-free variant of asd_lmhead_margin (the paper has no counterpart;
+ * this is a library convenience).  Same arguments and outputs, but instead
+ * of a caller-provided workspace it uses scratch memory that the library
+ * reserves statically: a device array of ASD_NOALLOC_SCRATCH_BYTES that every
+ * GPU which loads libasd holds until the process exits.  It is meant for
+ * callers that cannot allocate device memory themselves, for example a plugin
+ * inside a serving engine that has reserved all free device memory for its
+ * own KV-cache pool, or a latency-critical loop where cudaMalloc (which may
+ * synchronise the device) is not acceptable.  The call itself allocates
+ * nothing.
+ *  - The first call on a device, with that device current, looks up the
+ *    array's device address; make that first call before any stream capture.
+ *  - Requests whose scratch needs exceed ASD_NOALLOC_SCRATCH_BYTES return
+ *    ASD_ERR_WORKSPACE without enqueuing anything (about 3,400 tree nodes on a
+ *    152-SM GB300: the scratch holds 16 bytes per node per SM plus 32 bytes
+ *    per node).
+ *  - All calls share the one array per device and it keeps the last call's
+ *    contents; every call clears what must start at zero.  Calls that overlap
+ *    on the GPU (different streams without ordering) race on the scratch and
+ *    must not be issued.
+ *  - device_status (optional device int32, may be NULL) receives the call's
+ *    device-side status word (asd_status) at the end of the enqueued work.
+ */
+#define ASD_NOALLOC_SCRATCH_BYTES (8u << 20)
+asd_status asd_lmhead_margin_noalloc(const asd_dims* dims, const void* hidden, const void* w_lm,
+                                     const int32_t* tokens, const int32_t* parent,
+                                     const int32_t* cu_nodes, int32_t total_nodes, float tau,
+                                     float* row_max, int32_t* row_argmax, float* row_lse,
+                                     float* l_draft, float* ratio, uint8_t* accept,
+                                     int32_t* device_status, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

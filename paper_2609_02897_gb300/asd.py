@@ -27,7 +27,7 @@ STATUS = {0: "ASD_OK", 1: "ASD_ERR_INVALID_ARG", 2: "ASD_ERR_SHAPE", 3: "ASD_ERR
           7: "ASD_ERR_CUDA", 8: "ASD_ERR_TIMEOUT", 9: "ASD_ERR_UNSUPPORTED"}
 EXPORTS = ["asd_workspace_bytes", "asd_tree_attention", "asd_lmhead_margin", "asd_accept_path",
            "asd_kv_compact", "asd_verify_step", "asd_get_device_status", "asd_status_string",
-           "asd_abi_version"]
+           "asd_abi_version", "asd_lmhead_margin_noalloc"]
 
 
 class AsdError(RuntimeError):
@@ -79,6 +79,9 @@ _lib.asd_kv_compact.argtypes = [_P, _vp, _vp, _vp, ctypes.c_int32] + [_vp] * 7 +
     _vp, ctypes.c_size_t, _vp]
 _lib.asd_verify_step.restype = ctypes.c_int
 _lib.asd_verify_step.argtypes = [_P, ctypes.POINTER(VerifyArgs), _vp, ctypes.c_size_t, _vp]
+_lib.asd_lmhead_margin_noalloc.restype = ctypes.c_int
+_lib.asd_lmhead_margin_noalloc.argtypes = [_P] + [_vp] * 5 + [ctypes.c_int32, ctypes.c_float] + [
+    _vp] * 6 + [_vp, _vp]
 _lib.asd_get_device_status.restype = ctypes.c_int
 _lib.asd_get_device_status.argtypes = [_vp, ctypes.POINTER(ctypes.c_int32), _vp]
 
@@ -145,6 +148,19 @@ def asd_lmhead_margin(dims, hidden, w_lm, tokens, parent, cu_nodes, tau, row_max
         int(parent.numel()), float(tau), _ptr(row_max), _ptr(row_argmax), _ptr(row_lse),
         _ptr(l_draft), _ptr(ratio), _ptr(accept), _ptr(workspace), workspace.numel(),
         _stream(stream)), "asd_lmhead_margin")
+
+
+def asd_lmhead_margin_noalloc(dims, hidden, w_lm, tokens, parent, cu_nodes, tau, row_max,
+                              row_argmax, row_lse, l_draft, ratio, accept, device_status=None,
+                              stream=None):
+    """asd_lmhead_margin with the library's static scratch instead of a workspace
+    (for callers that cannot allocate device memory).  device_status: optional
+    int32 device tensor that receives the device-side status word."""
+    _check(_lib.asd_lmhead_margin_noalloc(
+        ctypes.byref(dims), _ptr(hidden), _ptr(w_lm), _ptr(tokens), _ptr(parent), _ptr(cu_nodes),
+        int(parent.numel()), float(tau), _ptr(row_max), _ptr(row_argmax), _ptr(row_lse),
+        _ptr(l_draft), _ptr(ratio), _ptr(accept), _ptr(device_status), _stream(stream)),
+        "asd_lmhead_margin_noalloc")
 
 
 def asd_accept_path(dims, parent, tokens, accept, row_argmax, cu_nodes, path, path_len, bonus,

@@ -503,3 +503,103 @@ asd_status asd_get_device_status(const void* workspace, int32_t* status_out, voi
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------
+// Allocation-free LM head (asd_lmhead_margin_noalloc).  For callers that may
+// not allocate device memory (an engine that owns all free memory, a loop
+// that cannot afford cudaMalloc's implicit synchronisation), the scratch of
+// the LM-head path lives in this file-scope device array instead of a
+// caller-provided workspace.  Host code must not hand `g_noalloc_scratch`
+// itself to a kernel: in host code that name is only a host-side stand-in.
+// The device address is looked up once per device with cudaGetSymbolAddress.
+// ---------------------------------------------------------------------------
+static __device__ __align__(256) uint8_t g_noalloc_scratch[ASD_NOALLOC_SCRATCH_BYTES];
+
+namespace {
+
+std::mutex g_noalloc_mutex;
+void* g_noalloc_ptr[128] = {nullptr};
+
+// Device address of the scratch array on the current device; set up on the
+// first call per device (this first call must precede any stream capture).
+void* noalloc_scratch() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 128) return nullptr;
+  std::lock_guard<std::mutex> lock(g_noalloc_mutex);
+  if (!g_noalloc_ptr[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess) return nullptr;
+    g_noalloc_ptr[dev] = p;
+  }
+  return g_noalloc_ptr[dev];
+}
+
+// Regions of the LM-head path only (no attention partials).
+WsLayout lmhead_only_layout(const asd_dims& d, int T, int nsm) {
+  WsLayout L{};
+  L.g_lm = std::max(1, std::min(nsm, (d.vocab + kLmBoxRows - 1) / kLmBoxRows));
+  size_t off = 0;
+  L.status = off;      off = align256(off + 16);
+  L.seq_flags = off;   off = align256(off + 4 * static_cast<size_t>(d.batch));
+  L.anc = off;         off = align256(off + 16 * static_cast<size_t>(T));
+  L.child_start = off; off = align256(off + 4 * static_cast<size_t>(T));
+  L.child_cnt = off;   off = align256(off + 4 * static_cast<size_t>(T));
+  L.child_tok = off;   off = align256(off + 4 * static_cast<size_t>(T));
+  L.child_id = off;    off = align256(off + 4 * static_cast<size_t>(T));
+  L.lm_part = off;     off = align256(off + sizeof(LmPartial) * static_cast<size_t>(T) * L.g_lm);
+  L.attn_lse = L.attn_o = off;
+  L.total = off;
+  return L;
+}
+
+}  // namespace
+
+extern "C" asd_status asd_lmhead_margin_noalloc(
+    const asd_dims* dims, const void* hidden, const void* w_lm, const int32_t* tokens,
+    const int32_t* parent, const int32_t* cu_nodes, int32_t total_nodes, float tau,
+    float* row_max, int32_t* row_argmax, float* row_lse, float* l_draft, float* ratio,
+    uint8_t* accept, int32_t* device_status, void* stream) {
+  if (!hidden || !w_lm || !tokens || !parent || !cu_nodes || !row_max || !row_argmax ||
+      !row_lse || !l_draft || !ratio || !accept)
+    return ASD_ERR_INVALID_ARG;
+  if (!tau_ok(tau)) return ASD_ERR_INVALID_ARG;
+  if (!aligned16(hidden) || !aligned16(w_lm)) return ASD_ERR_INVALID_ARG;
+  if (!dims_ok(dims)) return dims ? ASD_ERR_SHAPE : ASD_ERR_INVALID_ARG;
+  if (!nodes_ok(dims, total_nodes)) return ASD_ERR_SHAPE;
+  const int nsm = device_sm_count();
+  if (nsm <= 0) return ASD_ERR_CUDA;
+  Ctx c;
+  c.d = *dims;
+  c.T = total_nodes;
+  c.L = lmhead_only_layout(*dims, total_nodes, nsm);
+  if (c.L.total > ASD_NOALLOC_SCRATCH_BYTES) return ASD_ERR_WORKSPACE;
+  c.ws = noalloc_scratch();
+  if (!c.ws) return ASD_ERR_CUDA;
+  c.st = static_cast<cudaStream_t>(stream);
+  // the status word must start at zero; every other region is written before it is read
+  if (cudaMemsetAsync(ws_at<int>(c.ws, c.L.status), 0, 16, c.st) != cudaSuccess)
+    return ASD_ERR_CUDA;
+  if (launch_tree_prep(prep_params(c, parent, tokens, cu_nodes, nullptr, l_draft), c.st) !=
+      cudaSuccess)
+    return ASD_ERR_CUDA;
+  asd_status st = run_lmhead(c, hidden, w_lm, l_draft);
+  if (st != ASD_OK) return st;
+  TailParams t = tail_params(c, kTailFinalize);
+  t.parent = parent;
+  t.tokens = tokens;
+  t.cu_nodes = cu_nodes;
+  t.seq_flags = ws_at<int>(c.ws, c.L.seq_flags);
+  t.ln_tau = ln_tau(tau);
+  t.row_max = row_max;
+  t.row_argmax = row_argmax;
+  t.row_lse = row_lse;
+  t.l_draft = l_draft;
+  t.ratio = ratio;
+  t.accept = accept;
+  if (launch_tail(t, c.st) != cudaSuccess) return ASD_ERR_CUDA;
+  if (device_status &&
+      cudaMemcpyAsync(device_status, ws_at<int>(c.ws, c.L.status), sizeof(int32_t),
+                      cudaMemcpyDeviceToDevice, c.st) != cudaSuccess)
+    return ASD_ERR_CUDA;
+  return ASD_OK;
+}
