@@ -33,7 +33,7 @@ METRIC = "verified tree nodes/s"
 UNIT = "nodes/s"
 CONFIG = 2
 TAU = 0.3
-N_STAGE_KERNELS = 5   # prep, attention, combine, LM head, tail
+N_STAGE_KERNELS = 4   # prep, attention (splits merged in-kernel), LM head, tail
 
 
 def parse():
@@ -280,23 +280,36 @@ def run_asd(args):
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize()
+    # timed region: K back-to-back steps; consecutive kernels overlap through
+    # programmatic dependent launch, so no events sit between them
     t_start.record(stream)
     for k in range(K):
-        for j in range(5):
-            step.args.stage_events[j] = evs[k][j].cuda_event
         step.run(stream)
     t_end.record(stream)
     torch.cuda.synchronize()
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize()
-    clk = clocks.stop()
     status = step.device_status()
     if status != 0:
         raise RuntimeError(f"device status {asd.STATUS.get(status, status)}")
     ms = t_start.elapsed_time(t_end) / K
+
+    # second timed region (same K): events at the stage boundaries of every
+    # step give each kernel's own duration; an event between two kernels
+    # serialises them, so this region is slower than the one above
+    torch.cuda.synchronize()
+    for k in range(K):
+        for j in range(5):
+            step.args.stage_events[j] = evs[k][j].cuda_event
+        step.run(stream)
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    for j in range(5):
+        step.args.stage_events[j] = None
     stage = np.array([[evs[k][j].elapsed_time(evs[k][j + 1]) for j in range(4)] for k in range(K)])
     stage_ms = stage.mean(axis=0)
+    staged_ms = float(np.mean([evs[k][0].elapsed_time(evs[k][4]) for k in range(K)]))
     lm_ms = float(stage_ms[2])
     if world > 1:
         t = torch.tensor([ms, lm_ms], device=device, dtype=torch.float64)
@@ -360,8 +373,10 @@ def run_asd(args):
                      "peak_source": peak_kind + " hbm_gbs (MEASURED_PEAKS.json)",
                      "algorithmic_bytes_per_launch": lmb, "avg_launch_us": 1e3 * lm_ms,
                      "traffic": None},
-        "stages_us": {"prep": 1e3 * stage_ms[0], "attention+combine": 1e3 * stage_ms[1],
-                      "lmhead": 1e3 * stage_ms[2], "tail": 1e3 * stage_ms[3]},
+        "stages_us": {"prep": 1e3 * stage_ms[0], "attention": 1e3 * stage_ms[1],
+                      "lmhead": 1e3 * stage_ms[2], "tail": 1e3 * stage_ms[3],
+                      "step_with_stage_events": 1e3 * staged_ms,
+                      "note": "second timed region with events between kernels (no overlap)"},
         "mean_path_len": mean_path,
         "gpu_launches": K * N_STAGE_KERNELS,
         "clocks": clk,

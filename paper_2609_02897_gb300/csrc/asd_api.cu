@@ -89,25 +89,27 @@ bool nodes_ok(const asd_dims* d, int32_t total_nodes) {
 WsLayout layout(const asd_dims& d, int T, int nsm) {
   WsLayout L{};
   const int G = d.num_q_heads / d.num_kv_heads;
-  L.g_lm = std::max(1, std::min(nsm, (d.vocab + kLmBoxRows - 1) / kLmBoxRows));
-  const int rblocks = (d.max_nodes * G + 63) / 64;
+  L.g_lm = std::max(1, std::min(std::min(nsm, kMaxLmRanges), (d.vocab + kLmBoxRows - 1) / kLmBoxRows));
+  // context splits: enough CTAs for about one wave at two CTAs per SM, at
+  // most kMaxAttnParts; the last non-empty split of a sequence also takes its
+  // tree keys, so there is no separate tree part
+  const int rblocks = attention_row_blocks(d.max_nodes, G);
   const long long base = static_cast<long long>(rblocks) * d.batch * d.num_kv_heads;
-  const long long target = 3LL * nsm;
-  if (d.ctx_max > 0) {
-    const int max_splits = (d.ctx_max + 63) / 64;
-    long long ns = (target + base - 1) / base;
-    ns = std::max(1LL, std::min(ns, static_cast<long long>(max_splits)));
-    const int per = static_cast<int>((d.ctx_max + ns - 1) / ns);
-    L.split_len = ((per + 63) / 64) * 64;
-    L.n_splits = (d.ctx_max + L.split_len - 1) / L.split_len;
-  } else {
-    L.split_len = 64;
-    L.n_splits = 0;
-  }
-  L.n_parts = L.n_splits + 1;
+  const long long target = 2LL * nsm;
+  const int max_splits = std::max(1, std::min(kMaxAttnParts, (d.ctx_max + 63) / 64));
+  long long ns = (target + base - 1) / base;
+  ns = std::max(1LL, std::min(ns, static_cast<long long>(max_splits)));
+  const int per = static_cast<int>((std::max(d.ctx_max, 1) + ns - 1) / ns);
+  L.split_len = ((per + 63) / 64) * 64;
+  L.n_splits = std::max(1, (d.ctx_max + L.split_len - 1) / L.split_len);
+  L.n_parts = L.n_splits;
   const size_t TH = static_cast<size_t>(T) * d.num_q_heads;
+  const size_t groups = static_cast<size_t>(d.batch) * d.num_kv_heads *
+                        attention_row_blocks(d.max_nodes, G);
   size_t off = 0;
   L.status = off;      off = align256(off + 16);
+  L.attn_cnt = off;    off = off + 4 * groups;
+  L.clear_bytes = off; off = align256(off);
   L.seq_flags = off;   off = align256(off + 4 * static_cast<size_t>(d.batch));
   L.anc = off;         off = align256(off + 16 * static_cast<size_t>(T));
   L.child_start = off; off = align256(off + 4 * static_cast<size_t>(T));
@@ -151,7 +153,7 @@ asd_status begin_call(const asd_dims* dims, int32_t total_nodes, void* ws, size_
   if (ws_bytes < c->L.total) return ASD_ERR_WORKSPACE;
   c->st = static_cast<cudaStream_t>(stream);
   c->ws = ws;
-  if (cudaMemsetAsync(ws_at<int>(ws, c->L.status), 0, 16, c->st) != cudaSuccess)
+  if (cudaMemsetAsync(ws_at<int>(ws, c->L.status), 0, c->L.clear_bytes, c->st) != cudaSuccess)
     return ASD_ERR_CUDA;
   return ASD_OK;
 }
@@ -196,6 +198,7 @@ asd_status run_attention(const Ctx& c, const void* q, const void* k_cache, const
   a.anc = ws_at<uint64_t>(c.ws, c.L.anc);
   a.part_o = ws_at<float>(c.ws, c.L.attn_o);
   a.part_lse = ws_at<float>(c.ws, c.L.attn_lse);
+  a.counters = ws_at<int>(c.ws, c.L.attn_cnt);
   a.status = ws_at<int>(c.ws, c.L.status);
   a.out = out;
   a.B = d.batch;
@@ -233,9 +236,7 @@ asd_status run_attention(const Ctx& c, const void* q, const void* k_cache, const
   } else {
     err = launch_attention_f32(a, c.st);
   }
-  if (err != cudaSuccess) return ASD_ERR_CUDA;
-  if (launch_attention_combine(a, d.dtype == ASD_BF16, c.st) != cudaSuccess) return ASD_ERR_CUDA;
-  return ASD_OK;
+  return err == cudaSuccess ? ASD_OK : ASD_ERR_CUDA;
 }
 
 asd_status run_lmhead(const Ctx& c, const void* hidden, const void* w, float* l_draft) {
@@ -537,7 +538,7 @@ void* noalloc_scratch() {
 // Regions of the LM-head path only (no attention partials).
 WsLayout lmhead_only_layout(const asd_dims& d, int T, int nsm) {
   WsLayout L{};
-  L.g_lm = std::max(1, std::min(nsm, (d.vocab + kLmBoxRows - 1) / kLmBoxRows));
+  L.g_lm = std::max(1, std::min(std::min(nsm, kMaxLmRanges), (d.vocab + kLmBoxRows - 1) / kLmBoxRows));
   size_t off = 0;
   L.status = off;      off = align256(off + 16);
   L.seq_flags = off;   off = align256(off + 4 * static_cast<size_t>(d.batch));
@@ -547,7 +548,8 @@ WsLayout lmhead_only_layout(const asd_dims& d, int T, int nsm) {
   L.child_tok = off;   off = align256(off + 4 * static_cast<size_t>(T));
   L.child_id = off;    off = align256(off + 4 * static_cast<size_t>(T));
   L.lm_part = off;     off = align256(off + sizeof(LmPartial) * static_cast<size_t>(T) * L.g_lm);
-  L.attn_lse = L.attn_o = off;
+  L.attn_lse = L.attn_o = L.attn_cnt = off;
+  L.clear_bytes = 16;
   L.total = off;
   return L;
 }

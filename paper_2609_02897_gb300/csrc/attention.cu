@@ -1,14 +1,16 @@
 // Tree attention of the verify pass (Sec. 2 "Verify": the target scores every
 // drafted node of the tree in one forward pass).
 //
-// Work unit: one CTA per (row block, sequence x KV head, split).  The query
-// rows of a (sequence, KV head) pair are its N nodes times the G query heads
-// that share the KV head (grouped-query attention), packed node-major:
-// row r -> node r / G, head g*G + r % G.  Splits 0..n_splits-1 cover slices of
-// the committed context (flash-decoding split-KV); split n_splits covers the
-// tree itself, where a node only sees its ancestors (bitmask from the tree
-// preparation kernel).  Each split writes its softmax-normalised partial
-// output and its log-sum-exp; the combine kernel merges the splits.
+// Work unit: one CTA per (row block, sequence x KV head, context split).  The
+// query rows of a (sequence, KV head) pair are its N nodes times the G query
+// heads that share the KV head (grouped-query attention), packed node-major:
+// row r -> node r / G, head g*G + r % G.  Split z covers context keys
+// [z*L, (z+1)*L) (flash-decoding split-KV); the CTA of the sequence's last
+// non-empty split also covers the tree keys, where a node only sees its
+// ancestors (bitmask from the tree preparation kernel).  Each split writes its
+// softmax-normalised partial output and its log-sum-exp; the last CTA of a
+// group to finish merges the group's splits into the output (atomic ticket,
+// no waiting).
 #include "kernels.h"
 
 namespace asd {
@@ -16,7 +18,7 @@ namespace {
 
 constexpr int kRowsPerCta = 64;   // 4 warps x 16 query rows
 constexpr int kKeysPerTile = 64;
-constexpr int kAttnStages = 2;  // 2 CTAs per SM fit with D = 128
+constexpr int kAttnStages = 2;    // 2 CTAs per SM fit with D = 128
 
 // ---------------------------------------------------------------- mma helpers
 __device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
@@ -68,6 +70,103 @@ struct RowMap {
   }
 };
 
+// Key range of one CTA: context keys [kbeg, kend) and, for the sequence's
+// last non-empty split (split 0 when the context is empty), the tree keys.
+struct KeyRange {
+  int kbeg, kend, nctx, ntree;
+  __device__ KeyRange(int z, int split_len, int ctx, int n) {
+    kbeg = z * split_len;
+    kend = min(kbeg + split_len, ctx);
+    nctx = kend > kbeg ? (kend - kbeg + kKeysPerTile - 1) / kKeysPerTile : 0;
+    const int last = ctx > 0 ? (ctx - 1) / split_len : 0;
+    ntree = (z == last) ? (n + kKeysPerTile - 1) / kKeysPerTile : 0;
+  }
+};
+
+// Called by every thread of a CTA once its split's rows are written.  The
+// last CTA of the (sequence, KV head, row block) group to arrive merges the
+// group's splits: out = sum_z 2^(lse_z - M) O_z / sum_z 2^(lse_z - M).  The
+// ticket is an atomic counter (zeroed by the host before the launch); no CTA
+// ever waits for another.  The merge first turns every row's log-sum-exps into
+// weights, then streams the split outputs part by part with every thread
+// holding kItems loads in flight.
+template <typename OutT, int D>
+__device__ __forceinline__ void finish_group(const AttnParams& p, const RowMap& rm, int nrows,
+                                             int group) {
+  constexpr int kC4 = D / 4;
+  constexpr int kItems = kRowsPerCta * kC4 / 128;
+  __shared__ int s_last;
+  __shared__ float s_w[kRowsPerCta][kMaxAttnParts];
+  __shared__ float s_inv[kRowsPerCta];
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) s_last = (atomicAdd(&p.counters[group], 1) == p.n_parts - 1);
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  const size_t TH = static_cast<size_t>(p.T) * p.Hq;
+  const int P = p.n_parts;
+  for (int r = threadIdx.x; r < nrows; r += blockDim.x) {
+    const size_t gr = rm.grow(r);
+    float l[kMaxAttnParts];
+    float M = -INFINITY;
+#pragma unroll
+    for (int zz = 0; zz < kMaxAttnParts; ++zz) {
+      l[zz] = zz < P ? __ldcg(p.part_lse + zz * TH + gr) : -INFINITY;
+      M = fmaxf(M, l[zz]);
+    }
+    float sum = 0.f;
+#pragma unroll
+    for (int zz = 0; zz < kMaxAttnParts; ++zz) {
+      const float w = (l[zz] == -INFINITY) ? 0.f : exp2f(l[zz] - M);
+      s_w[r][zz] = w;
+      sum += w;
+    }
+    s_inv[r] = sum > 0.f ? 1.f / sum : 0.f;
+  }
+  __syncthreads();
+  float4 acc[kItems];
+#pragma unroll
+  for (int k = 0; k < kItems; ++k) acc[k] = make_float4(0.f, 0.f, 0.f, 0.f);
+  // every split wrote finite rows (zeros for an empty split), so the loads of
+  // one part are unconditional and all kItems of them are in flight together
+  size_t row_off[kItems];
+#pragma unroll
+  for (int k = 0; k < kItems; ++k) {
+    const int it = threadIdx.x + 128 * k;
+    const int r = min(it / kC4, nrows - 1);
+    row_off[k] = rm.grow(r) * D + 4 * (it - (it / kC4) * kC4);
+  }
+  for (int zz = 0; zz < P; ++zz) {
+    const float* base = p.part_o + zz * TH * D;
+    float4 v[kItems];
+#pragma unroll
+    for (int k = 0; k < kItems; ++k) v[k] = __ldcg(reinterpret_cast<const float4*>(base + row_off[k]));
+#pragma unroll
+    for (int k = 0; k < kItems; ++k) {
+      const int it = threadIdx.x + 128 * k;
+      const float w = s_w[min(it / kC4, nrows - 1)][zz];
+      acc[k].x = fmaf(w, v[k].x, acc[k].x);
+      acc[k].y = fmaf(w, v[k].y, acc[k].y);
+      acc[k].z = fmaf(w, v[k].z, acc[k].z);
+      acc[k].w = fmaf(w, v[k].w, acc[k].w);
+    }
+  }
+#pragma unroll
+  for (int k = 0; k < kItems; ++k) {
+    const int it = threadIdx.x + 128 * k;
+    const int r = it / kC4, c4 = it - r * kC4;
+    if (r < nrows) {
+      const float inv = s_inv[r];
+      OutT* out = static_cast<OutT*>(p.out) + rm.grow(r) * D + 4 * c4;
+      out[0] = from_f32<OutT>(acc[k].x * inv);
+      out[1] = from_f32<OutT>(acc[k].y * inv);
+      out[2] = from_f32<OutT>(acc[k].z * inv);
+      out[3] = from_f32<OutT>(acc[k].w * inv);
+    }
+  }
+}
+
 // ----------------------------------------------------------- bf16 tensor path
 template <int D>
 __global__ void __launch_bounds__(128) attn_bf16_kernel(const __grid_constant__ CUtensorMap tm_k,
@@ -79,31 +178,25 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const __grid_constant__ 
   extern __shared__ uint8_t smem_raw[];
   __shared__ int s_abort;
 
+  pdl_launch_dependents();  // the LM head may start streaming its weights now
+
+  // The sequence extent and context length are caller inputs that the tree
+  // preparation kernel validates.  Before its verdict (pdl_wait below) this
+  // kernel only starts TMA copies of context K/V, whose coordinates stay
+  // inside the tensor maps whatever those inputs hold.
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int rb = blockIdx.x, bg = blockIdx.y, z = blockIdx.z;
   const int b = bg / p.Hkv, g = bg - b * p.Hkv;
-  if (p.seq_flags[b] & (kSeqBadTree | kSeqBadCtx)) return;
   const int s0 = p.cu_nodes[b];
   const int n = p.cu_nodes[b + 1] - s0;
   const int R = n * p.G;
   const int r0 = rb * kRowsPerCta;
-  if (r0 >= R) return;
+  if (n <= 0 || n > kMaxNodes || r0 >= R) return;
   const int nrows = min(kRowsPerCta, R - r0);
-  const bool is_tree = (z == p.n_splits);
-  int kbeg, kend;
-  if (is_tree) {
-    kbeg = 0;
-    kend = n;
-  } else {
-    kbeg = z * p.split_len;
-    kend = min(kbeg + p.split_len, p.ctx_len[b]);
-  }
+  const KeyRange kr(z, p.split_len, min(p.ctx_len[b], p.ctx_max), n);
   const RowMap rm{s0, p.G, p.Hq, g, r0};
   const size_t TH = static_cast<size_t>(p.T) * p.Hq;
-  if (kbeg >= kend) {
-    for (int r = tid; r < nrows; r += 128) p.part_lse[z * TH + rm.grow(r)] = -INFINITY;
-    return;
-  }
+  const int group = bg * gridDim.x + rb;
 
   uint32_t base = smem_u32(smem_raw);
   const uint32_t pad = (1024u - (base & 1023u)) & 1023u;
@@ -117,30 +210,12 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const __grid_constant__ 
   uint8_t* gK = smem + kTileBytes;
   uint8_t* gV = gK + kAttnStages * kTileBytes;
 
-  // query rows -> shared memory (swizzled like the TMA tiles)
-  const __nv_bfloat16* q = static_cast<const __nv_bfloat16*>(p.q);
-  for (int c = tid; c < kRowsPerCta * kChunks; c += 128) {
-    const int r = c / kChunks, ch = c - r * kChunks;
-    uint4 v = make_uint4(0u, 0u, 0u, 0u);
-    if (r < nrows) v = *reinterpret_cast<const uint4*>(q + rm.grow(r) * D + ch * 8);
-    *reinterpret_cast<uint4*>(gQ + sw_off(r, ch)) = v;
-  }
-  if (tid == 0) {
-    s_abort = 0;
-    if (!is_tree) {
-      for (int s = 0; s < kAttnStages; ++s) mbar_init(sBar + 8 * s, 1);
-      fence_mbar_init();
-    }
-  }
-  __syncthreads();
-
-  const int ntiles = (kend - kbeg + kKeysPerTile - 1) / kKeysPerTile;
   const int ps = p.page_size;
   uint64_t pol = 0;
 
   auto issue = [&](int t) {
     const int stage = t % kAttnStages;
-    const int key0 = kbeg + t * kKeysPerTile;
+    const int key0 = kr.kbeg + t * kKeysPerTile;
     const uint32_t dK = sK + stage * kTileBytes, dV = sV + stage * kTileBytes;
     const uint32_t bar = sBar + 8 * stage;
     if (ps == 0) {
@@ -154,12 +229,12 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const __grid_constant__ 
     } else {
       const int br = ps < 64 ? ps : 64;  // rows per box
       const int nbox = kKeysPerTile / br;
-      int rows[kKeysPerTile / 8];  // at most 8 boxes (page_size >= 8)
+      int rows[kKeysPerTile / 8];        // at most 8 boxes (page_size >= 8)
       int cnt = 0;
       for (int j = 0; j < nbox; ++j) {
         const int key = key0 + j * br;
         rows[j] = -1;
-        if (key >= kend) continue;
+        if (key >= kr.kend) continue;
         const int page = p.page_table[static_cast<size_t>(b) * p.pages_per_seq + key / ps];
         if (page < 0 || page >= p.num_pages) {
           set_status(p.status, ASD_ERR_CTX_RANGE);
@@ -180,12 +255,49 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const __grid_constant__ 
     }
   };
 
-  if (!is_tree && tid == 0) {
-    pol = l2_policy_evict_first();
-    prefetch_tmap(&tm_k);
-    prefetch_tmap(&tm_v);
-    for (int t = 0; t < ntiles && t < kAttnStages; ++t) issue(t);
+  // the producer thread sets up the barriers and starts the first K/V tiles
+  // before waiting for the tree preparation and staging the query rows
+  if (tid == 0) {
+    s_abort = 0;
+    if (kr.nctx > 0) {
+      for (int s = 0; s < kAttnStages; ++s) mbar_init(sBar + 8 * s, 1);
+      fence_mbar_init();
+      pol = l2_policy_evict_first();
+      prefetch_tmap(&tm_k);
+      prefetch_tmap(&tm_v);
+      for (int t = 0; t < kr.nctx && t < kAttnStages; ++t) issue(t);
+    }
   }
+
+  pdl_wait();  // tree preparation results: sequence flags, ancestor masks
+  if (p.seq_flags[b] & (kSeqBadTree | kSeqBadCtx)) {
+    // skip the sequence, but only after the copies already started have landed
+    if (tid == 0)
+      for (int t = 0; t < kr.nctx && t < kAttnStages; ++t) mbar_wait(sBar + 8 * t, 0);
+    __syncthreads();
+    return;
+  }
+  if (kr.nctx + kr.ntree == 0) {
+    // empty split: weight-zero log-sum-exp and finite (zero) rows for the merge
+    for (int r = tid; r < nrows; r += 128) p.part_lse[z * TH + rm.grow(r)] = -INFINITY;
+    for (int idx = tid; idx < nrows * (D / 4); idx += 128) {
+      const int r = idx / (D / 4), c4 = idx - r * (D / 4);
+      *reinterpret_cast<float4*>(p.part_o + (z * TH + rm.grow(r)) * D + 4 * c4) =
+          make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+    finish_group<__nv_bfloat16, D>(p, rm, nrows, group);
+    return;
+  }
+
+  // query rows -> shared memory (swizzled like the TMA tiles)
+  const __nv_bfloat16* q = static_cast<const __nv_bfloat16*>(p.q);
+  for (int c = tid; c < kRowsPerCta * kChunks; c += 128) {
+    const int r = c / kChunks, ch = c - r * kChunks;
+    uint4 v = make_uint4(0u, 0u, 0u, 0u);
+    if (r < nrows) v = *reinterpret_cast<const uint4*>(q + rm.grow(r) * D + ch * 8);
+    *reinterpret_cast<uint4*>(gQ + sw_off(r, ch)) = v;
+  }
+  __syncthreads();
 
   // Q fragments stay in registers for the whole kernel
   uint32_t qa[D / 16][4];
@@ -196,10 +308,10 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const __grid_constant__ 
     ldsm_x4(sQ + sw_off(row, chunk), qa[ks][0], qa[ks][1], qa[ks][2], qa[ks][3]);
   }
 
-  // ancestor masks of this thread's two rows (tree split)
+  // ancestor masks of this thread's two rows (tree tiles only)
   const int rowA = warp * 16 + (lane >> 2), rowB = rowA + 8;
   uint64_t aAlo = 0, aAhi = 0, aBlo = 0, aBhi = 0;
-  if (is_tree) {
+  if (kr.ntree > 0) {
     if (rowA < nrows) {
       const int node = s0 + (r0 + rowA) / p.G;
       aAlo = p.anc[2 * node];
@@ -221,13 +333,15 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const __grid_constant__ 
   const __nv_bfloat16* tk = static_cast<const __nv_bfloat16*>(p.tree_k);
   const __nv_bfloat16* tv = static_cast<const __nv_bfloat16*>(p.tree_v);
 
+  const int ntiles = kr.nctx + kr.ntree;
   for (int t = 0; t < ntiles; ++t) {
     const int stage = t % kAttnStages;
-    const int key0 = kbeg + t * kKeysPerTile;
-    const int valid = min(kKeysPerTile, kend - key0);
+    const bool tree_tile = t >= kr.nctx;
+    const int key0 = tree_tile ? (t - kr.nctx) * kKeysPerTile : kr.kbeg + t * kKeysPerTile;
+    const int valid = min(kKeysPerTile, (tree_tile ? n : kr.kend) - key0);
     uint8_t* gKs = gK + stage * kTileBytes;
     uint8_t* gVs = gV + stage * kTileBytes;
-    if (is_tree) {
+    if (tree_tile) {
       for (int cidx = tid; cidx < kKeysPerTile * kChunks; cidx += 128) {
         const int r = cidx / kChunks, ch = cidx - r * kChunks;
         uint4 kv = make_uint4(0u, 0u, 0u, 0u), vv = kv;
@@ -278,13 +392,10 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const __grid_constant__ 
 #pragma unroll
       for (int e = 0; e < 2; ++e) {
         const int local = 8 * j + 2 * kq + e;
-        bool vA, vB;
-        if (is_tree) {
-          const int key = key0 + local;
-          vA = key < kend && anc_bit(aAlo, aAhi, key);
-          vB = key < kend && anc_bit(aBlo, aBhi, key);
-        } else {
-          vA = vB = local < valid;
+        bool vA = local < valid, vB = vA;
+        if (tree_tile) {
+          vA = vA && anc_bit(aAlo, aAhi, key0 + local);
+          vB = vB && anc_bit(aBlo, aBhi, key0 + local);
         }
         sc[j][e] = vA ? sc[j][e] : -INFINITY;
         sc[j][2 + e] = vB ? sc[j][2 + e] : -INFINITY;
@@ -340,7 +451,7 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const __grid_constant__ 
       }
     }
     __syncthreads();  // every warp is done with this stage
-    if (!is_tree && tid == 0 && t + kAttnStages < ntiles) {
+    if (tid == 0 && t + kAttnStages < kr.nctx) {
       fence_proxy_async();
       issue(t + kAttnStages);
     }
@@ -368,6 +479,7 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const __grid_constant__ 
       *reinterpret_cast<float2*>(dst + 8 * j + 2 * kq) = make_float2(o[j][2] * iB, o[j][3] * iB);
     if (kq == 0) p.part_lse[z * TH + gr] = (mB == -INFINITY) ? -INFINITY : mB * c + log2f(lB);
   }
+  finish_group<__nv_bfloat16, D>(p, rm, nrows, group);
 }
 
 // ----------------------------------------------------------- fp32 SIMT path
@@ -376,6 +488,8 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const __grid_constant__ 
 template <int D>
 __global__ void __launch_bounds__(128) attn_f32_kernel(const AttnParams p) {
   constexpr int kPer = D / 32;
+  pdl_wait();
+  pdl_launch_dependents();
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int rb = blockIdx.x, bg = blockIdx.y, z = blockIdx.z;
   const int b = bg / p.Hkv, g = bg - b * p.Hkv;
@@ -386,15 +500,7 @@ __global__ void __launch_bounds__(128) attn_f32_kernel(const AttnParams p) {
   const int r0 = rb * kRowsPerCta;
   if (r0 >= R) return;
   const int nrows = min(kRowsPerCta, R - r0);
-  const bool is_tree = (z == p.n_splits);
-  int kbeg, kend;
-  if (is_tree) {
-    kbeg = 0;
-    kend = n;
-  } else {
-    kbeg = z * p.split_len;
-    kend = min(kbeg + p.split_len, p.ctx_len[b]);
-  }
+  const KeyRange kr(z, p.split_len, min(p.ctx_len[b], p.ctx_max), n);
   const RowMap rm{s0, p.G, p.Hq, g, r0};
   const size_t TH = static_cast<size_t>(p.T) * p.Hq;
   const float* qp = static_cast<const float*>(p.q);
@@ -404,11 +510,16 @@ __global__ void __launch_bounds__(128) attn_f32_kernel(const AttnParams p) {
   const float* tv = static_cast<const float*>(p.tree_v);
   const float c = p.scale_log2;
   const int ps = p.page_size;
+  const int nctx_keys = max(0, kr.kend - kr.kbeg);
+  const int ntree_keys = kr.ntree > 0 ? n : 0;
 
   for (int r = warp; r < nrows; r += 4) {
     const size_t gr = rm.grow(r);
-    if (kbeg >= kend) {
+    if (nctx_keys + ntree_keys == 0) {
+      // empty split: weight-zero log-sum-exp and a finite (zero) row
       if (lane == 0) p.part_lse[z * TH + gr] = -INFINITY;
+#pragma unroll
+      for (int k = 0; k < kPer; ++k) p.part_o[(z * TH + gr) * D + lane + 32 * k] = 0.f;
       continue;
     }
     float qv[kPer], ov[kPer];
@@ -418,37 +529,40 @@ __global__ void __launch_bounds__(128) attn_f32_kernel(const AttnParams p) {
       ov[k] = 0.f;
     }
     uint64_t alo = 0, ahi = 0;
-    if (is_tree) {
+    if (ntree_keys) {
       const int node = s0 + (r0 + r) / p.G;
       alo = p.anc[2 * node];
       ahi = p.anc[2 * node + 1];
     }
     float m = -INFINITY, l = 0.f;
-    for (int key = kbeg; key < kend; ++key) {
-      const float* kr;
+    for (int t = 0; t < nctx_keys + ntree_keys; ++t) {
+      const float* kr_;
       const float* vr;
-      if (is_tree) {
+      if (t >= nctx_keys) {
+        const int key = t - nctx_keys;
         if (!anc_bit(alo, ahi, key)) continue;
         const size_t off = (static_cast<size_t>(s0 + key) * p.Hkv + g) * D;
-        kr = tk + off;
+        kr_ = tk + off;
         vr = tv + off;
       } else if (ps == 0) {
+        const int key = kr.kbeg + t;
         const size_t off = ((static_cast<size_t>(b) * p.Hkv + g) * p.ctx_max + key) * D;
-        kr = kc + off;
+        kr_ = kc + off;
         vr = vc + off;
       } else {
+        const int key = kr.kbeg + t;
         const int page = p.page_table[static_cast<size_t>(b) * p.pages_per_seq + key / ps];
         if (page < 0 || page >= p.num_pages) {
           if (lane == 0) set_status(p.status, ASD_ERR_CTX_RANGE);
           continue;
         }
         const size_t off = ((static_cast<size_t>(page) * p.Hkv + g) * ps + key % ps) * D;
-        kr = kc + off;
+        kr_ = kc + off;
         vr = vc + off;
       }
       float dot = 0.f;
 #pragma unroll
-      for (int k = 0; k < kPer; ++k) dot = fmaf(qv[k], kr[lane + 32 * k], dot);
+      for (int k = 0; k < kPer; ++k) dot = fmaf(qv[k], kr_[lane + 32 * k], dot);
 #pragma unroll
       for (int off = 16; off > 0; off >>= 1) dot += __shfl_xor_sync(0xffffffffu, dot, off);
       const float mn = fmaxf(m, dot);
@@ -465,46 +579,7 @@ __global__ void __launch_bounds__(128) attn_f32_kernel(const AttnParams p) {
     for (int k = 0; k < kPer; ++k) dst[lane + 32 * k] = ov[k] * inv;
     if (lane == 0) p.part_lse[z * TH + gr] = (m == -INFINITY) ? -INFINITY : m * c + log2f(l);
   }
-}
-
-// -------------------------------------------------------------------- combine
-template <typename OutT, int D>
-__global__ void __launch_bounds__(128) attn_combine_kernel(const AttnParams p) {
-  constexpr int kPer = D / 32;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const size_t TH = static_cast<size_t>(p.T) * p.Hq;
-  const size_t row = static_cast<size_t>(blockIdx.x) * 4 + warp;
-  if (row >= TH) return;
-  float M = -INFINITY;
-  for (int zz = 0; zz < p.n_parts; ++zz) M = fmaxf(M, p.part_lse[zz * TH + row]);
-  float acc[kPer];
-#pragma unroll
-  for (int k = 0; k < kPer; ++k) acc[k] = 0.f;
-  float wsum = 0.f;
-  if (M != -INFINITY) {
-    for (int zz = 0; zz < p.n_parts; ++zz) {
-      const float lz = p.part_lse[zz * TH + row];
-      if (lz == -INFINITY) continue;
-      const float w = exp2f(lz - M);
-      wsum += w;
-      const float* src = p.part_o + (zz * TH + row) * D + lane * kPer;
-      if constexpr (kPer == 4) {
-        const float4 v = *reinterpret_cast<const float4*>(src);
-        acc[0] = fmaf(w, v.x, acc[0]);
-        acc[1] = fmaf(w, v.y, acc[1]);
-        acc[2] = fmaf(w, v.z, acc[2]);
-        acc[3] = fmaf(w, v.w, acc[3]);
-      } else {
-        const float2 v = *reinterpret_cast<const float2*>(src);
-        acc[0] = fmaf(w, v.x, acc[0]);
-        acc[1] = fmaf(w, v.y, acc[1]);
-      }
-    }
-  }
-  const float inv = wsum > 0.f ? 1.f / wsum : 0.f;
-  OutT* out = static_cast<OutT*>(p.out) + row * D + lane * kPer;
-#pragma unroll
-  for (int k = 0; k < kPer; ++k) out[k] = from_f32<OutT>(acc[k] * inv);
+  finish_group<float, D>(p, rm, nrows, bg * gridDim.x + rb);
 }
 
 }  // namespace
@@ -514,48 +589,34 @@ size_t attn_bf16_smem_bytes(int D) {
   return 1024 + tile * (1 + 2 * kAttnStages) + 8 * kAttnStages;
 }
 
+int attention_row_blocks(int max_nodes, int G) {
+  return (max_nodes * G + kRowsPerCta - 1) / kRowsPerCta;
+}
+
 static dim3 attn_grid(const AttnParams& p) {
-  const int rblocks = (p.max_nodes * p.G + kRowsPerCta - 1) / kRowsPerCta;
-  return dim3(rblocks, p.B * p.Hkv, p.n_parts);
+  return dim3(attention_row_blocks(p.max_nodes, p.G), p.B * p.Hkv, p.n_parts);
 }
 
 cudaError_t launch_attention_bf16(const AttnParams& p, const CUtensorMap& tm_k,
                                   const CUtensorMap& tm_v, cudaStream_t s) {
   const size_t smem = attn_bf16_smem_bytes(p.D);
-  cudaError_t err;
   if (p.D == 128) {
-    err = cudaFuncSetAttribute(attn_bf16_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                               static_cast<int>(smem));
+    cudaError_t err = cudaFuncSetAttribute(attn_bf16_kernel<128>,
+                                           cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                           static_cast<int>(smem));
     if (err != cudaSuccess) return err;
-    attn_bf16_kernel<128><<<attn_grid(p), 128, smem, s>>>(tm_k, tm_v, p);
-  } else {
-    err = cudaFuncSetAttribute(attn_bf16_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                               static_cast<int>(smem));
-    if (err != cudaSuccess) return err;
-    attn_bf16_kernel<64><<<attn_grid(p), 128, smem, s>>>(tm_k, tm_v, p);
+    return launch_pdl(attn_bf16_kernel<128>, attn_grid(p), dim3(128), smem, s, tm_k, tm_v, p);
   }
-  return cudaGetLastError();
+  cudaError_t err = cudaFuncSetAttribute(attn_bf16_kernel<64>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(smem));
+  if (err != cudaSuccess) return err;
+  return launch_pdl(attn_bf16_kernel<64>, attn_grid(p), dim3(128), smem, s, tm_k, tm_v, p);
 }
 
 cudaError_t launch_attention_f32(const AttnParams& p, cudaStream_t s) {
-  if (p.D == 128)
-    attn_f32_kernel<128><<<attn_grid(p), 128, 0, s>>>(p);
-  else
-    attn_f32_kernel<64><<<attn_grid(p), 128, 0, s>>>(p);
-  return cudaGetLastError();
-}
-
-cudaError_t launch_attention_combine(const AttnParams& p, bool bf16, cudaStream_t s) {
-  const size_t rows = static_cast<size_t>(p.T) * p.Hq;
-  const dim3 grid(static_cast<unsigned>((rows + 3) / 4));
-  if (bf16) {
-    if (p.D == 128) attn_combine_kernel<__nv_bfloat16, 128><<<grid, 128, 0, s>>>(p);
-    else attn_combine_kernel<__nv_bfloat16, 64><<<grid, 128, 0, s>>>(p);
-  } else {
-    if (p.D == 128) attn_combine_kernel<float, 128><<<grid, 128, 0, s>>>(p);
-    else attn_combine_kernel<float, 64><<<grid, 128, 0, s>>>(p);
-  }
-  return cudaGetLastError();
+  if (p.D == 128) return launch_pdl(attn_f32_kernel<128>, attn_grid(p), dim3(128), 0, s, p);
+  return launch_pdl(attn_f32_kernel<64>, attn_grid(p), dim3(128), 0, s, p);
 }
 
 }  // namespace asd

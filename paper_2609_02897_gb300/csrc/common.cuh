@@ -11,6 +11,8 @@
 namespace asd {
 
 constexpr int kMaxNodes = ASD_MAX_TREE_NODES;
+constexpr int kMaxLmRanges = 256;   // upper bound on LM-head vocabulary ranges (CTAs)
+constexpr int kMaxAttnParts = 32;   // upper bound on attention context splits
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
 // Bounded waits give up after this many SM clock cycles (about 2 s at 2 GHz).
@@ -30,6 +32,8 @@ struct LmPartial {
 // Offsets (bytes) of the workspace regions; every region is 256-byte aligned.
 struct WsLayout {
   size_t status;       // int32[4]: [0] first device error code
+  size_t attn_cnt;     // int32[B*Hkv*row_blocks]: split tickets of the attention groups
+  size_t clear_bytes;  // bytes from offset 0 that every call zeroes (status + tickets)
   size_t seq_flags;    // int32[B]
   size_t anc;          // uint64[T][2]: ancestor bitmask of each node (self included)
   size_t child_start;  // int32[T]: global slot of the node's first child
@@ -50,6 +54,16 @@ struct WsLayout {
 
 __device__ __forceinline__ void set_status(int* status, int code) {
   atomicCAS(status, 0, code);
+}
+
+// Programmatic dependent launch: a kernel launched with programmatic stream
+// serialisation may start while its predecessor in the stream still runs;
+// pdl_wait() blocks until every predecessor grid has completed and its memory
+// is visible, pdl_launch_dependents() lets the next kernel start launching.
+// Both are no-ops for kernels launched without the attribute.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 }
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {

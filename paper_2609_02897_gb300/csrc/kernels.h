@@ -5,9 +5,29 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <utility>
+
 #include "common.cuh"
 
 namespace asd {
+
+// Launches `kernel` with programmatic stream serialisation, so it may begin
+// while the previous kernel in the stream finishes (see pdl_wait()).
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                       cudaStream_t s, Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
 
 // ------------------------------------------------------------ tree preparation
 struct PrepParams {
@@ -41,6 +61,7 @@ struct AttnParams {
   const uint64_t* anc;
   float* part_o;            // [n_parts][T*Hq][D]
   float* part_lse;          // [n_parts][T*Hq]
+  int* counters;            // [B*Hkv*row_blocks] split tickets, zero on entry
   int* status;
   void* out;                // [T, Hq, D]
   int B, T, Hq, Hkv, G, D;
@@ -50,10 +71,11 @@ struct AttnParams {
 };
 // bf16 path: tensor-core (mma.sync) split-KV kernel fed by TMA; tm_k / tm_v are
 // 2D tensor maps over the context cache rows (box 64 x min(64, rows per page)).
+// Both paths merge their splits in-kernel (the last CTA of each group).
 cudaError_t launch_attention_bf16(const AttnParams& p, const CUtensorMap& tm_k,
                                   const CUtensorMap& tm_v, cudaStream_t s);
 cudaError_t launch_attention_f32(const AttnParams& p, cudaStream_t s);
-cudaError_t launch_attention_combine(const AttnParams& p, bool bf16, cudaStream_t s);
+int attention_row_blocks(int max_nodes, int G);
 
 // -------------------------------------------------------------------- LM head
 struct LmParams {

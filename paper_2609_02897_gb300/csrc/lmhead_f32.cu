@@ -15,6 +15,8 @@ constexpr int kKc = 32;      // hidden elements staged per step
 __global__ void __launch_bounds__(kRows) lmhead_f32_kernel(const LmParams p) {
   __shared__ float s_w[32][kKc + 1];
   __shared__ float s_h[kRows][kKc + 1];
+  pdl_wait();
+  pdl_launch_dependents();
   const int tid = threadIdx.x;
   const float* hid = static_cast<const float*>(p.hidden);
   const float* w = static_cast<const float*>(p.w);
@@ -72,8 +74,7 @@ __global__ void __launch_bounds__(kRows) lmhead_f32_kernel(const LmParams p) {
 }  // namespace
 
 cudaError_t launch_lmhead_f32(const LmParams& p, cudaStream_t s) {
-  lmhead_f32_kernel<<<p.g_lm, kRows, 0, s>>>(p);
-  return cudaGetLastError();
+  return launch_pdl(lmhead_f32_kernel, dim3(p.g_lm), dim3(kRows), 0, s, p);
 }
 
 }  // namespace asd

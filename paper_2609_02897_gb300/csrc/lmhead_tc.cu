@@ -113,6 +113,9 @@ __global__ void __launch_bounds__(192, 1)
   __shared__ uint32_t s_tmem;
   __shared__ volatile int s_abort;
 
+  // W and the hidden states are inputs of the step, not results of earlier
+  // kernels: only the epilogue (children lists, l_draft) waits for them
+  pdl_launch_dependents();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
   // this CTA's vocabulary range, in whole groups of kLmBoxRows rows
@@ -248,6 +251,7 @@ __global__ void __launch_bounds__(192, 1)
     // ----------------------------------------------------------------- epilogue
     const int q = warp & 3;
     const int row = q * 32 + lane;
+    pdl_wait();
     int acc = 0;
     uint32_t aph = 0;
     bool ok = true;
@@ -313,8 +317,7 @@ cudaError_t launch_lmhead_bf16(const LmParams& p, const CUtensorMap& tm_hidden,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(smem));
   if (err != cudaSuccess) return err;
-  lmhead_tc_kernel<<<p.g_lm, 192, smem, s>>>(tm_hidden, tm_w, p);
-  return cudaGetLastError();
+  return launch_pdl(lmhead_tc_kernel, dim3(p.g_lm), dim3(192), smem, s, tm_hidden, tm_w, p);
 }
 
 }  // namespace asd

@@ -1,5 +1,5 @@
-// Per-sequence tail of the verify step, one CTA of 128 threads per sequence
-// (thread i owns local node i).  Three stages, selected by TailParams::mode:
+// Per-sequence tail of the verify step, one CTA of 1024 threads per sequence
+// (thread i < N owns local node i; all 32 warps share the merge and the copy).  Three stages, selected by TailParams::mode:
 //  finalize  merge the LM head's per-range partials of every row into
 //            row_max / row_argmax / row_lse and evaluate the margin rule for
 //            every drafted node: ratio = exp(l_draft - row_max[parent]) (Eq. 1),
@@ -18,6 +18,9 @@
 namespace asd {
 namespace {
 
+constexpr int kTailThreads = 1024;     // 32 warps: one node's merge per warp
+constexpr int kMaxPartsPerLane = kMaxLmRanges / 32;
+
 __device__ __forceinline__ void merge_part(float& m, float& s, int& a, float m2, float s2,
                                            int a2) {
   if (m2 == -INFINITY) return;
@@ -34,7 +37,7 @@ __device__ __forceinline__ void merge_part(float& m, float& s, int& a, float m2,
   m = M;
 }
 
-__global__ void __launch_bounds__(kMaxNodes) tail_kernel(const TailParams p) {
+__global__ void __launch_bounds__(kTailThreads) tail_kernel(const TailParams p) {
   __shared__ int s_par[kMaxNodes];
   __shared__ int s_tok[kMaxNodes];
   __shared__ int s_arg[kMaxNodes];
@@ -46,6 +49,7 @@ __global__ void __launch_bounds__(kMaxNodes) tail_kernel(const TailParams p) {
   __shared__ int s_path[kMaxNodes];
   __shared__ int s_maxd, s_len, s_skip;
 
+  pdl_wait();  // every earlier kernel of the step has completed
   const int b = blockIdx.x;
   const int i = threadIdx.x;
   const int warp = i >> 5, lane = i & 31;
@@ -86,14 +90,20 @@ __global__ void __launch_bounds__(kMaxNodes) tail_kernel(const TailParams p) {
   // ---------------------------------------------------------------- finalize
   if (p.mode & kTailFinalize) {
     if (!tree_bad) {
-      for (int r = warp; r < n; r += 4) {
+      // one warp per node: every lane loads its (up to 8) partials before merging
+      for (int r = warp; r < n; r += kTailThreads / 32) {
         const size_t node = static_cast<size_t>(s + r);
+        const float4* src = reinterpret_cast<const float4*>(p.part + node * p.g_lm);
+        float4 q[kMaxPartsPerLane];
+#pragma unroll
+        for (int k = 0; k < kMaxPartsPerLane; ++k) {
+          const int g = lane + 32 * k;
+          q[k] = g < p.g_lm ? __ldcg(src + g) : make_float4(-INFINITY, 0.f, 0.f, 0.f);
+        }
         float m = -INFINITY, sm = 0.f;
         int a = INT_MAX;
-        for (int g = lane; g < p.g_lm; g += 32) {
-          const LmPartial q = p.part[node * p.g_lm + g];
-          merge_part(m, sm, a, q.m, q.s, q.a);
-        }
+#pragma unroll
+        for (int k = 0; k < kMaxPartsPerLane; ++k) merge_part(m, sm, a, q[k].x, q[k].y, __float_as_int(q[k].z));
 #pragma unroll
         for (int off = 16; off > 0; off >>= 1) {
           const float m2 = __shfl_xor_sync(0xffffffffu, m, off);
@@ -173,10 +183,10 @@ __global__ void __launch_bounds__(kMaxNodes) tail_kernel(const TailParams p) {
         p.n_promoted[b] = len > 0 ? promoted : 0;
       }
       __syncthreads();
-      for (int k = i; k < p.max_path; k += kMaxNodes)
+      for (int k = i; k < p.max_path; k += kTailThreads)
         p.path[static_cast<size_t>(b) * p.max_path + k] = k < s_len ? s_path[k] : -1;
     } else {
-      for (int k = i; k < p.max_path; k += kMaxNodes)
+      for (int k = i; k < p.max_path; k += kTailThreads)
         p.path[static_cast<size_t>(b) * p.max_path + k] = -1;
       if (i == 0) {
         p.path_len[b] = 0;
@@ -221,7 +231,7 @@ __global__ void __launch_bounds__(kMaxNodes) tail_kernel(const TailParams p) {
     const uint8_t* tv = static_cast<const uint8_t*>(p.tree_v);
     uint8_t* kc = static_cast<uint8_t*>(p.k_cache);
     uint8_t* vc = static_cast<uint8_t*>(p.v_cache);
-    for (int idx = i; idx < len * per_node; idx += kMaxNodes) {
+    for (int idx = i; idx < len * per_node; idx += kTailThreads) {
       const int k = idx / per_node;
       const int rem = idx - k * per_node;
       const int g = rem / chunks;
@@ -250,8 +260,7 @@ __global__ void __launch_bounds__(kMaxNodes) tail_kernel(const TailParams p) {
 }  // namespace
 
 cudaError_t launch_tail(const TailParams& p, cudaStream_t s) {
-  tail_kernel<<<p.B, kMaxNodes, 0, s>>>(p);
-  return cudaGetLastError();
+  return launch_pdl(tail_kernel, dim3(p.B), dim3(kTailThreads), 0, s, p);
 }
 
 }  // namespace asd

@@ -18,6 +18,7 @@ __global__ void __launch_bounds__(kMaxNodes) tree_prep_kernel(PrepParams p) {
   __shared__ int s_start[kMaxNodes];
   __shared__ int s_bad;
 
+  pdl_launch_dependents();
   const int b = blockIdx.x;
   const int i = threadIdx.x;
   const int s = p.cu_nodes[b];
