@@ -91,8 +91,8 @@ WsLayout layout(const asd_dims& d, int T, int nsm) {
   const int G = d.num_q_heads / d.num_kv_heads;
   L.g_lm = std::max(1, std::min(std::min(nsm, kMaxLmRanges), (d.vocab + kLmBoxRows - 1) / kLmBoxRows));
   // context splits: enough CTAs for about one wave at two CTAs per SM, at
-  // most kMaxAttnParts; the last non-empty split of a sequence also takes its
-  // tree keys, so there is no separate tree part
+  // most kMaxAttnParts (the splits of a row block form one thread-block
+  // cluster); the last non-empty split of a sequence also takes its tree keys
   const int rblocks = attention_row_blocks(d.max_nodes, G);
   const long long base = static_cast<long long>(rblocks) * d.batch * d.num_kv_heads;
   const long long target = 2LL * nsm;
@@ -103,13 +103,8 @@ WsLayout layout(const asd_dims& d, int T, int nsm) {
   L.split_len = ((per + 63) / 64) * 64;
   L.n_splits = std::max(1, (d.ctx_max + L.split_len - 1) / L.split_len);
   L.n_parts = L.n_splits;
-  const size_t TH = static_cast<size_t>(T) * d.num_q_heads;
-  const size_t groups = static_cast<size_t>(d.batch) * d.num_kv_heads *
-                        attention_row_blocks(d.max_nodes, G);
   size_t off = 0;
   L.status = off;      off = align256(off + 16);
-  L.attn_cnt = off;    off = off + 4 * groups;
-  L.clear_bytes = off; off = align256(off);
   L.seq_flags = off;   off = align256(off + 4 * static_cast<size_t>(d.batch));
   L.anc = off;         off = align256(off + 16 * static_cast<size_t>(T));
   L.child_start = off; off = align256(off + 4 * static_cast<size_t>(T));
@@ -117,8 +112,6 @@ WsLayout layout(const asd_dims& d, int T, int nsm) {
   L.child_tok = off;   off = align256(off + 4 * static_cast<size_t>(T));
   L.child_id = off;    off = align256(off + 4 * static_cast<size_t>(T));
   L.lm_part = off;     off = align256(off + sizeof(LmPartial) * static_cast<size_t>(T) * L.g_lm);
-  L.attn_lse = off;    off = align256(off + 4 * L.n_parts * TH);
-  L.attn_o = off;      off = align256(off + 4 * L.n_parts * TH * d.head_dim);
   L.total = off;
   return L;
 }
@@ -153,7 +146,7 @@ asd_status begin_call(const asd_dims* dims, int32_t total_nodes, void* ws, size_
   if (ws_bytes < c->L.total) return ASD_ERR_WORKSPACE;
   c->st = static_cast<cudaStream_t>(stream);
   c->ws = ws;
-  if (cudaMemsetAsync(ws_at<int>(ws, c->L.status), 0, c->L.clear_bytes, c->st) != cudaSuccess)
+  if (cudaMemsetAsync(ws_at<int>(ws, c->L.status), 0, 16, c->st) != cudaSuccess)
     return ASD_ERR_CUDA;
   return ASD_OK;
 }
@@ -196,9 +189,6 @@ asd_status run_attention(const Ctx& c, const void* q, const void* k_cache, const
   a.page_table = page_table;
   a.seq_flags = ws_at<int>(c.ws, c.L.seq_flags);
   a.anc = ws_at<uint64_t>(c.ws, c.L.anc);
-  a.part_o = ws_at<float>(c.ws, c.L.attn_o);
-  a.part_lse = ws_at<float>(c.ws, c.L.attn_lse);
-  a.counters = ws_at<int>(c.ws, c.L.attn_cnt);
   a.status = ws_at<int>(c.ws, c.L.status);
   a.out = out;
   a.B = d.batch;
@@ -548,8 +538,6 @@ WsLayout lmhead_only_layout(const asd_dims& d, int T, int nsm) {
   L.child_tok = off;   off = align256(off + 4 * static_cast<size_t>(T));
   L.child_id = off;    off = align256(off + 4 * static_cast<size_t>(T));
   L.lm_part = off;     off = align256(off + sizeof(LmPartial) * static_cast<size_t>(T) * L.g_lm);
-  L.attn_lse = L.attn_o = L.attn_cnt = off;
-  L.clear_bytes = 16;
   L.total = off;
   return L;
 }

@@ -7,10 +7,12 @@
 // row r -> node r / G, head g*G + r % G.  Split z covers context keys
 // [z*L, (z+1)*L) (flash-decoding split-KV); the CTA of the sequence's last
 // non-empty split also covers the tree keys, where a node only sees its
-// ancestors (bitmask from the tree preparation kernel).  Each split writes its
-// softmax-normalised partial output and its log-sum-exp; the last CTA of a
-// group to finish merges the group's splits into the output (atomic ticket,
-// no waiting).
+// ancestors (bitmask from the tree preparation kernel).  The splits of one
+// (row block, sequence x KV head) form a thread-block cluster: each CTA keeps
+// its softmax-normalised partial output and log-sum-exp in shared memory, and
+// after a cluster barrier every CTA merges a slice of the rows by reading its
+// peers' partials through distributed shared memory.  No partial leaves the
+// cluster.
 #include "kernels.h"
 
 namespace asd {
@@ -83,88 +85,103 @@ struct KeyRange {
   }
 };
 
-// Called by every thread of a CTA once its split's rows are written.  The
-// last CTA of the (sequence, KV head, row block) group to arrive merges the
-// group's splits: out = sum_z 2^(lse_z - M) O_z / sum_z 2^(lse_z - M).  The
-// ticket is an atomic counter (zeroed by the host before the launch); no CTA
-// ever waits for another.  The merge first turns every row's log-sum-exps into
-// weights, then streams the split outputs part by part with every thread
-// holding kItems loads in flight.
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;"
+               ::: "memory");
+}
+
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+
+// Address of the same shared-memory location in cluster CTA `rank`.
+__device__ __forceinline__ uint32_t peer_addr(uint32_t local, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(local), "r"(rank));
+  return r;
+}
+
+__device__ __forceinline__ float ld_peer_f32(uint32_t addr) {
+  float v;
+  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(addr) : "memory");
+  return v;
+}
+
+__device__ __forceinline__ float4 ld_peer_f4(uint32_t addr) {
+  float4 v;
+  asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
+               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+               : "r"(addr)
+               : "memory");
+  return v;
+}
+
+// Merge of the cluster's splits.  Every CTA of the cluster holds, for its
+// rows, the split output normalised by its own softmax sum in s_o[r][D]
+// (fp32) and the split's log2-domain log-sum-exp in s_lse[r] (-inf for an
+// empty split, whose rows are zero).  After a cluster barrier, CTA `rank`
+// merges rows [rank*per, (rank+1)*per):
+//   out = sum_z 2^(lse_z - M) O_z / sum_z 2^(lse_z - M),
+// reading its peers' shared memory; a second barrier keeps every CTA alive
+// until its peers are done reading.
 template <typename OutT, int D>
-__device__ __forceinline__ void finish_group(const AttnParams& p, const RowMap& rm, int nrows,
-                                             int group) {
+__device__ __forceinline__ void cluster_merge(const AttnParams& p, const RowMap& rm, int nrows,
+                                              uint32_t s_o, uint32_t s_lse) {
   constexpr int kC4 = D / 4;
-  constexpr int kItems = kRowsPerCta * kC4 / 128;
-  __shared__ int s_last;
   __shared__ float s_w[kRowsPerCta][kMaxAttnParts];
   __shared__ float s_inv[kRowsPerCta];
-  __threadfence();
-  __syncthreads();
-  if (threadIdx.x == 0) s_last = (atomicAdd(&p.counters[group], 1) == p.n_parts - 1);
-  __syncthreads();
-  if (!s_last) return;
-  __threadfence();
-  const size_t TH = static_cast<size_t>(p.T) * p.Hq;
+  cluster_sync();
   const int P = p.n_parts;
-  for (int r = threadIdx.x; r < nrows; r += blockDim.x) {
-    const size_t gr = rm.grow(r);
+  const uint32_t rank = cluster_rank();
+  const int per = (nrows + P - 1) / P;
+  const int rbeg = static_cast<int>(rank) * per;
+  const int rend = min(nrows, rbeg + per);
+  for (int r = rbeg + static_cast<int>(threadIdx.x); r < rend; r += blockDim.x) {
     float l[kMaxAttnParts];
     float M = -INFINITY;
 #pragma unroll
     for (int zz = 0; zz < kMaxAttnParts; ++zz) {
-      l[zz] = zz < P ? __ldcg(p.part_lse + zz * TH + gr) : -INFINITY;
+      l[zz] = zz < P ? ld_peer_f32(peer_addr(s_lse + 4 * r, zz)) : -INFINITY;
       M = fmaxf(M, l[zz]);
     }
     float sum = 0.f;
 #pragma unroll
     for (int zz = 0; zz < kMaxAttnParts; ++zz) {
       const float w = (l[zz] == -INFINITY) ? 0.f : exp2f(l[zz] - M);
-      s_w[r][zz] = w;
+      s_w[r - rbeg][zz] = w;
       sum += w;
     }
-    s_inv[r] = sum > 0.f ? 1.f / sum : 0.f;
+    s_inv[r - rbeg] = sum > 0.f ? 1.f / sum : 0.f;
   }
   __syncthreads();
-  float4 acc[kItems];
+  for (int it = threadIdx.x; it < (rend - rbeg) * kC4; it += blockDim.x) {
+    const int rl = it / kC4, c4 = it - rl * kC4;
+    const uint32_t off = s_o + static_cast<uint32_t>(((rbeg + rl) * D + 4 * c4) * 4);
+    float4 v[kMaxAttnParts];
 #pragma unroll
-  for (int k = 0; k < kItems; ++k) acc[k] = make_float4(0.f, 0.f, 0.f, 0.f);
-  // every split wrote finite rows (zeros for an empty split), so the loads of
-  // one part are unconditional and all kItems of them are in flight together
-  size_t row_off[kItems];
+    for (int zz = 0; zz < kMaxAttnParts; ++zz)
+      if (zz < P) v[zz] = ld_peer_f4(peer_addr(off, zz));
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
-  for (int k = 0; k < kItems; ++k) {
-    const int it = threadIdx.x + 128 * k;
-    const int r = min(it / kC4, nrows - 1);
-    row_off[k] = rm.grow(r) * D + 4 * (it - (it / kC4) * kC4);
-  }
-  for (int zz = 0; zz < P; ++zz) {
-    const float* base = p.part_o + zz * TH * D;
-    float4 v[kItems];
-#pragma unroll
-    for (int k = 0; k < kItems; ++k) v[k] = __ldcg(reinterpret_cast<const float4*>(base + row_off[k]));
-#pragma unroll
-    for (int k = 0; k < kItems; ++k) {
-      const int it = threadIdx.x + 128 * k;
-      const float w = s_w[min(it / kC4, nrows - 1)][zz];
-      acc[k].x = fmaf(w, v[k].x, acc[k].x);
-      acc[k].y = fmaf(w, v[k].y, acc[k].y);
-      acc[k].z = fmaf(w, v[k].z, acc[k].z);
-      acc[k].w = fmaf(w, v[k].w, acc[k].w);
+    for (int zz = 0; zz < kMaxAttnParts; ++zz) {
+      if (zz < P) {
+        const float w = s_w[rl][zz];
+        acc.x = fmaf(w, v[zz].x, acc.x);
+        acc.y = fmaf(w, v[zz].y, acc.y);
+        acc.z = fmaf(w, v[zz].z, acc.z);
+        acc.w = fmaf(w, v[zz].w, acc.w);
+      }
     }
+    const float inv = s_inv[rl];
+    OutT* out = static_cast<OutT*>(p.out) + rm.grow(rbeg + rl) * D + 4 * c4;
+    out[0] = from_f32<OutT>(acc.x * inv);
+    out[1] = from_f32<OutT>(acc.y * inv);
+    out[2] = from_f32<OutT>(acc.z * inv);
+    out[3] = from_f32<OutT>(acc.w * inv);
   }
-#pragma unroll
-  for (int k = 0; k < kItems; ++k) {
-    const int it = threadIdx.x + 128 * k;
-    const int r = it / kC4, c4 = it - r * kC4;
-    if (r < nrows) {
-      const float inv = s_inv[r];
-      OutT* out = static_cast<OutT*>(p.out) + rm.grow(r) * D + 4 * c4;
-      out[0] = from_f32<OutT>(acc[k].x * inv);
-      out[1] = from_f32<OutT>(acc[k].y * inv);
-      out[2] = from_f32<OutT>(acc[k].z * inv);
-      out[3] = from_f32<OutT>(acc[k].w * inv);
-    }
-  }
+  cluster_sync();
 }
 
 // ----------------------------------------------------------- bf16 tensor path
@@ -177,6 +194,7 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const __grid_constant__ 
   constexpr int kChunks = D / 8;
   extern __shared__ uint8_t smem_raw[];
   __shared__ int s_abort;
+  __shared__ float s_lse[kRowsPerCta];
 
   pdl_launch_dependents();  // the LM head may start streaming its weights now
 
@@ -195,8 +213,6 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const __grid_constant__ 
   const int nrows = min(kRowsPerCta, R - r0);
   const KeyRange kr(z, p.split_len, min(p.ctx_len[b], p.ctx_max), n);
   const RowMap rm{s0, p.G, p.Hq, g, r0};
-  const size_t TH = static_cast<size_t>(p.T) * p.Hq;
-  const int group = bg * gridDim.x + rb;
 
   uint32_t base = smem_u32(smem_raw);
   const uint32_t pad = (1024u - (base & 1023u)) & 1023u;
@@ -277,15 +293,13 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const __grid_constant__ 
     __syncthreads();
     return;
   }
+  // after the tile loop the K stages hold this split's fp32 output rows
+  float* s_o = reinterpret_cast<float*>(gK);
   if (kr.nctx + kr.ntree == 0) {
     // empty split: weight-zero log-sum-exp and finite (zero) rows for the merge
-    for (int r = tid; r < nrows; r += 128) p.part_lse[z * TH + rm.grow(r)] = -INFINITY;
-    for (int idx = tid; idx < nrows * (D / 4); idx += 128) {
-      const int r = idx / (D / 4), c4 = idx - r * (D / 4);
-      *reinterpret_cast<float4*>(p.part_o + (z * TH + rm.grow(r)) * D + 4 * c4) =
-          make_float4(0.f, 0.f, 0.f, 0.f);
-    }
-    finish_group<__nv_bfloat16, D>(p, rm, nrows, group);
+    for (int r = tid; r < kRowsPerCta; r += 128) s_lse[r] = -INFINITY;
+    for (int idx = tid; idx < kRowsPerCta * D; idx += 128) s_o[idx] = 0.f;
+    cluster_merge<__nv_bfloat16, D>(p, rm, nrows, sK, smem_u32(s_lse));
     return;
   }
 
@@ -456,30 +470,26 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const __grid_constant__ 
       issue(t + kAttnStages);
     }
   }
-  if (s_abort) return;
+  if (s_abort) {  // a bounded wait gave up: contribute nothing, still meet the cluster
+    mA = mB = -INFINITY;
+    lA = lB = 0.f;
+  }
 
   lA += __shfl_xor_sync(0xffffffffu, lA, 1);
   lA += __shfl_xor_sync(0xffffffffu, lA, 2);
   lB += __shfl_xor_sync(0xffffffffu, lB, 1);
   lB += __shfl_xor_sync(0xffffffffu, lB, 2);
   const float iA = lA > 0.f ? 1.f / lA : 0.f, iB = lB > 0.f ? 1.f / lB : 0.f;
-  if (rowA < nrows) {
-    const size_t gr = rm.grow(rowA);
-    float* dst = p.part_o + (z * TH + gr) * D;
 #pragma unroll
-    for (int j = 0; j < D / 8; ++j)
-      *reinterpret_cast<float2*>(dst + 8 * j + 2 * kq) = make_float2(o[j][0] * iA, o[j][1] * iA);
-    if (kq == 0) p.part_lse[z * TH + gr] = (mA == -INFINITY) ? -INFINITY : mA * c + log2f(lA);
+  for (int j = 0; j < D / 8; ++j) {
+    *reinterpret_cast<float2*>(s_o + rowA * D + 8 * j + 2 * kq) = make_float2(o[j][0] * iA, o[j][1] * iA);
+    *reinterpret_cast<float2*>(s_o + rowB * D + 8 * j + 2 * kq) = make_float2(o[j][2] * iB, o[j][3] * iB);
   }
-  if (rowB < nrows) {
-    const size_t gr = rm.grow(rowB);
-    float* dst = p.part_o + (z * TH + gr) * D;
-#pragma unroll
-    for (int j = 0; j < D / 8; ++j)
-      *reinterpret_cast<float2*>(dst + 8 * j + 2 * kq) = make_float2(o[j][2] * iB, o[j][3] * iB);
-    if (kq == 0) p.part_lse[z * TH + gr] = (mB == -INFINITY) ? -INFINITY : mB * c + log2f(lB);
+  if (kq == 0) {
+    s_lse[rowA] = (mA == -INFINITY) ? -INFINITY : mA * c + log2f(lA);
+    s_lse[rowB] = (mB == -INFINITY) ? -INFINITY : mB * c + log2f(lB);
   }
-  finish_group<__nv_bfloat16, D>(p, rm, nrows, group);
+  cluster_merge<__nv_bfloat16, D>(p, rm, nrows, sK, smem_u32(s_lse));
 }
 
 // ----------------------------------------------------------- fp32 SIMT path
@@ -488,6 +498,9 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const __grid_constant__ 
 template <int D>
 __global__ void __launch_bounds__(128) attn_f32_kernel(const AttnParams p) {
   constexpr int kPer = D / 32;
+  extern __shared__ __align__(16) uint8_t smem_raw[];
+  __shared__ float s_lse[kRowsPerCta];
+  float* s_o = reinterpret_cast<float*>(smem_raw);   // [64][D] split output rows
   pdl_wait();
   pdl_launch_dependents();
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -502,7 +515,6 @@ __global__ void __launch_bounds__(128) attn_f32_kernel(const AttnParams p) {
   const int nrows = min(kRowsPerCta, R - r0);
   const KeyRange kr(z, p.split_len, min(p.ctx_len[b], p.ctx_max), n);
   const RowMap rm{s0, p.G, p.Hq, g, r0};
-  const size_t TH = static_cast<size_t>(p.T) * p.Hq;
   const float* qp = static_cast<const float*>(p.q);
   const float* kc = static_cast<const float*>(p.k_cache);
   const float* vc = static_cast<const float*>(p.v_cache);
@@ -517,9 +529,9 @@ __global__ void __launch_bounds__(128) attn_f32_kernel(const AttnParams p) {
     const size_t gr = rm.grow(r);
     if (nctx_keys + ntree_keys == 0) {
       // empty split: weight-zero log-sum-exp and a finite (zero) row
-      if (lane == 0) p.part_lse[z * TH + gr] = -INFINITY;
+      if (lane == 0) s_lse[r] = -INFINITY;
 #pragma unroll
-      for (int k = 0; k < kPer; ++k) p.part_o[(z * TH + gr) * D + lane + 32 * k] = 0.f;
+      for (int k = 0; k < kPer; ++k) s_o[r * D + lane + 32 * k] = 0.f;
       continue;
     }
     float qv[kPer], ov[kPer];
@@ -574,12 +586,11 @@ __global__ void __launch_bounds__(128) attn_f32_kernel(const AttnParams p) {
       m = mn;
     }
     const float inv = l > 0.f ? 1.f / l : 0.f;
-    float* dst = p.part_o + (z * TH + gr) * D;
 #pragma unroll
-    for (int k = 0; k < kPer; ++k) dst[lane + 32 * k] = ov[k] * inv;
-    if (lane == 0) p.part_lse[z * TH + gr] = (m == -INFINITY) ? -INFINITY : m * c + log2f(l);
+    for (int k = 0; k < kPer; ++k) s_o[r * D + lane + 32 * k] = ov[k] * inv;
+    if (lane == 0) s_lse[r] = (m == -INFINITY) ? -INFINITY : m * c + log2f(l);
   }
-  finish_group<float, D>(p, rm, nrows, bg * gridDim.x + rb);
+  cluster_merge<float, D>(p, rm, nrows, smem_u32(s_o), smem_u32(s_lse));
 }
 
 }  // namespace
@@ -597,6 +608,27 @@ static dim3 attn_grid(const AttnParams& p) {
   return dim3(attention_row_blocks(p.max_nodes, p.G), p.B * p.Hkv, p.n_parts);
 }
 
+// The n_parts splits of one (row block, sequence x KV head) form a cluster.
+template <typename... KArgs, typename... Args>
+static cudaError_t launch_attn(void (*kernel)(KArgs...), const AttnParams& p, size_t smem,
+                               cudaStream_t s, Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = attn_grid(p);
+  cfg.blockDim = dim3(128);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 1;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = static_cast<unsigned>(p.n_parts);
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 2;
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
+
 cudaError_t launch_attention_bf16(const AttnParams& p, const CUtensorMap& tm_k,
                                   const CUtensorMap& tm_v, cudaStream_t s) {
   const size_t smem = attn_bf16_smem_bytes(p.D);
@@ -605,18 +637,19 @@ cudaError_t launch_attention_bf16(const AttnParams& p, const CUtensorMap& tm_k,
                                            cudaFuncAttributeMaxDynamicSharedMemorySize,
                                            static_cast<int>(smem));
     if (err != cudaSuccess) return err;
-    return launch_pdl(attn_bf16_kernel<128>, attn_grid(p), dim3(128), smem, s, tm_k, tm_v, p);
+    return launch_attn(attn_bf16_kernel<128>, p, smem, s, tm_k, tm_v, p);
   }
   cudaError_t err = cudaFuncSetAttribute(attn_bf16_kernel<64>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(smem));
   if (err != cudaSuccess) return err;
-  return launch_pdl(attn_bf16_kernel<64>, attn_grid(p), dim3(128), smem, s, tm_k, tm_v, p);
+  return launch_attn(attn_bf16_kernel<64>, p, smem, s, tm_k, tm_v, p);
 }
 
 cudaError_t launch_attention_f32(const AttnParams& p, cudaStream_t s) {
-  if (p.D == 128) return launch_pdl(attn_f32_kernel<128>, attn_grid(p), dim3(128), 0, s, p);
-  return launch_pdl(attn_f32_kernel<64>, attn_grid(p), dim3(128), 0, s, p);
+  const size_t smem = static_cast<size_t>(kRowsPerCta) * p.D * sizeof(float);
+  if (p.D == 128) return launch_attn(attn_f32_kernel<128>, p, smem, s, p);
+  return launch_attn(attn_f32_kernel<64>, p, smem, s, p);
 }
 
 }  // namespace asd

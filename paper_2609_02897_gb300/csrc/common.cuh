@@ -12,7 +12,7 @@ namespace asd {
 
 constexpr int kMaxNodes = ASD_MAX_TREE_NODES;
 constexpr int kMaxLmRanges = 256;   // upper bound on LM-head vocabulary ranges (CTAs)
-constexpr int kMaxAttnParts = 32;   // upper bound on attention context splits
+constexpr int kMaxAttnParts = 8;    // attention context splits = cluster size (portable max)
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
 // Bounded waits give up after this many SM clock cycles (about 2 s at 2 GHz).
@@ -32,8 +32,6 @@ struct LmPartial {
 // Offsets (bytes) of the workspace regions; every region is 256-byte aligned.
 struct WsLayout {
   size_t status;       // int32[4]: [0] first device error code
-  size_t attn_cnt;     // int32[B*Hkv*row_blocks]: split tickets of the attention groups
-  size_t clear_bytes;  // bytes from offset 0 that every call zeroes (status + tickets)
   size_t seq_flags;    // int32[B]
   size_t anc;          // uint64[T][2]: ancestor bitmask of each node (self included)
   size_t child_start;  // int32[T]: global slot of the node's first child
@@ -41,13 +39,11 @@ struct WsLayout {
   size_t child_tok;    // int32[T]: children tokens, grouped by parent, sorted by (token, id)
   size_t child_id;     // int32[T]: global node id of each slot
   size_t lm_part;      // LmPartial[T][g_lm]
-  size_t attn_lse;     // float[n_parts][T*Hq]: log2-domain log-sum-exp per split
-  size_t attn_o;       // float[n_parts][T*Hq][D]: split outputs normalised per split
   size_t total;
   int g_lm;            // CTAs of the LM-head kernel (vocabulary ranges)
   int n_splits;        // context splits of the attention kernel
   int split_len;       // keys per context split (multiple of 64)
-  int n_parts;         // n_splits + 1 (the tree part)
+  int n_parts;         // = n_splits (the tree keys ride with the last split)
 };
 
 // ---------------------------------------------------------------- device utils

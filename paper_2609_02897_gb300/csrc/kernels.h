@@ -59,9 +59,6 @@ struct AttnParams {
   const int32_t* page_table;  // [B, ctx_max / ps] or null
   const int* seq_flags;
   const uint64_t* anc;
-  float* part_o;            // [n_parts][T*Hq][D]
-  float* part_lse;          // [n_parts][T*Hq]
-  int* counters;            // [B*Hkv*row_blocks] split tickets, zero on entry
   int* status;
   void* out;                // [T, Hq, D]
   int B, T, Hq, Hkv, G, D;
@@ -71,7 +68,7 @@ struct AttnParams {
 };
 // bf16 path: tensor-core (mma.sync) split-KV kernel fed by TMA; tm_k / tm_v are
 // 2D tensor maps over the context cache rows (box 64 x min(64, rows per page)).
-// Both paths merge their splits in-kernel (the last CTA of each group).
+// Both paths merge the splits of a group inside its thread-block cluster.
 cudaError_t launch_attention_bf16(const AttnParams& p, const CUtensorMap& tm_k,
                                   const CUtensorMap& tm_v, cudaStream_t s);
 cudaError_t launch_attention_f32(const AttnParams& p, cudaStream_t s);
