@@ -106,7 +106,6 @@ WsLayout layout(const asd_dims& d, int T, int nsm) {
   size_t off = 0;
   L.status = off;      off = align256(off + 16);
   L.seq_flags = off;   off = align256(off + 4 * static_cast<size_t>(d.batch));
-  L.anc = off;         off = align256(off + 16 * static_cast<size_t>(T));
   L.child_start = off; off = align256(off + 4 * static_cast<size_t>(T));
   L.child_cnt = off;   off = align256(off + 4 * static_cast<size_t>(T));
   L.child_tok = off;   off = align256(off + 4 * static_cast<size_t>(T));
@@ -160,7 +159,6 @@ PrepParams prep_params(const Ctx& c, const int32_t* parent, const int32_t* token
   p.ctx_len = ctx_len;
   p.status = ws_at<int>(c.ws, c.L.status);
   p.seq_flags = ws_at<int>(c.ws, c.L.seq_flags);
-  p.anc = ws_at<uint64_t>(c.ws, c.L.anc);
   p.child_start = ws_at<int32_t>(c.ws, c.L.child_start);
   p.child_cnt = ws_at<int32_t>(c.ws, c.L.child_cnt);
   p.child_tok = ws_at<int32_t>(c.ws, c.L.child_tok);
@@ -176,7 +174,8 @@ PrepParams prep_params(const Ctx& c, const int32_t* parent, const int32_t* token
 
 asd_status run_attention(const Ctx& c, const void* q, const void* k_cache, const void* v_cache,
                          const int32_t* page_table, const int32_t* ctx_len, const void* tree_k,
-                         const void* tree_v, const int32_t* cu, void* out) {
+                         const void* tree_v, const int32_t* parent, const int32_t* cu,
+                         void* out) {
   const asd_dims& d = c.d;
   AttnParams a{};
   a.q = q;
@@ -187,8 +186,7 @@ asd_status run_attention(const Ctx& c, const void* q, const void* k_cache, const
   a.cu_nodes = cu;
   a.ctx_len = ctx_len;
   a.page_table = page_table;
-  a.seq_flags = ws_at<int>(c.ws, c.L.seq_flags);
-  a.anc = ws_at<uint64_t>(c.ws, c.L.anc);
+  a.parent = parent;
   a.status = ws_at<int>(c.ws, c.L.status);
   a.out = out;
   a.B = d.batch;
@@ -245,10 +243,11 @@ asd_status run_lmhead(const Ctx& c, const void* hidden, const void* w, float* l_
   p.K = d.hidden;
   p.V = d.vocab;
   p.g_lm = c.L.g_lm;
+  p.a_rows = std::min(128, (c.T + 7) / 8 * 8);
   cudaError_t err;
   if (d.dtype == ASD_BF16) {
     CUtensorMap th, tw;
-    if (!make_tmap_bf16(&th, hidden, d.hidden, c.T, 128) ||
+    if (!make_tmap_bf16(&th, hidden, d.hidden, c.T, static_cast<uint32_t>(p.a_rows)) ||
         !make_tmap_bf16(&tw, w, d.hidden, d.vocab, kLmBoxRows))
       return ASD_ERR_CUDA;
     err = launch_lmhead_bf16(p, th, tw, c.st);
@@ -334,7 +333,8 @@ asd_status asd_tree_attention(const asd_dims* dims, const void* q, const void* k
   if (launch_tree_prep(prep_params(c, parent, nullptr, cu_nodes, ctx_len, nullptr), c.st) !=
       cudaSuccess)
     return ASD_ERR_CUDA;
-  return run_attention(c, q, k_cache, v_cache, page_table, ctx_len, tree_k, tree_v, cu_nodes, out);
+  return run_attention(c, q, k_cache, v_cache, page_table, ctx_len, tree_k, tree_v, parent,
+                       cu_nodes, out);
 }
 
 asd_status asd_lmhead_margin(const asd_dims* dims, const void* hidden, const void* w_lm,
@@ -448,7 +448,7 @@ asd_status asd_verify_step(const asd_dims* dims, const asd_verify_args* a, void*
     return ASD_ERR_CUDA;
   record(a->stage_events[1], c.st);
   st = run_attention(c, a->q, a->k_cache, a->v_cache, a->page_table, a->ctx_len, a->tree_k,
-                     a->tree_v, a->cu_nodes, a->attn_out);
+                     a->tree_v, a->parent, a->cu_nodes, a->attn_out);
   if (st != ASD_OK) return st;
   record(a->stage_events[2], c.st);
   st = run_lmhead(c, a->hidden, a->w_lm, a->l_draft);
@@ -532,7 +532,6 @@ WsLayout lmhead_only_layout(const asd_dims& d, int T, int nsm) {
   size_t off = 0;
   L.status = off;      off = align256(off + 16);
   L.seq_flags = off;   off = align256(off + 4 * static_cast<size_t>(d.batch));
-  L.anc = off;         off = align256(off + 16 * static_cast<size_t>(T));
   L.child_start = off; off = align256(off + 4 * static_cast<size_t>(T));
   L.child_cnt = off;   off = align256(off + 4 * static_cast<size_t>(T));
   L.child_tok = off;   off = align256(off + 4 * static_cast<size_t>(T));

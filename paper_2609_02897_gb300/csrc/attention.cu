@@ -63,6 +63,28 @@ __device__ __forceinline__ bool anc_bit(uint64_t lo, uint64_t hi, int j) {
   return j < 64 ? ((lo >> j) & 1ull) : ((hi >> (j - 64)) & 1ull);
 }
 
+// Ancestor bitmasks (self included) of the nodes of one tree, computed by
+// walking the parent array in shared memory.  Malformed entries (the tree
+// preparation kernel reports them) end the walk, so the loop is bounded.
+__device__ __forceinline__ void tree_ancestors(const int32_t* parent, int s0, int n, int* s_par,
+                                               uint64_t (*s_anc)[2]) {
+  for (int i = threadIdx.x; i < n; i += blockDim.x) s_par[i] = parent[s0 + i];
+  __syncthreads();
+  for (int i = threadIdx.x; i < n; i += blockDim.x) {
+    uint64_t lo = 0, hi = 0;
+    int u = i;
+    while (true) {
+      if (u < 64) lo |= 1ull << u; else hi |= 1ull << (u - 64);
+      const int pu = s_par[u];
+      if (pu < 0 || pu >= u) break;
+      u = pu;
+    }
+    s_anc[i][0] = lo;
+    s_anc[i][1] = hi;
+  }
+  __syncthreads();
+}
+
 struct RowMap {
   int s0, G, Hq, g, r0;
   __device__ __forceinline__ size_t grow(int r) const {
@@ -195,13 +217,15 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const __grid_constant__ 
   extern __shared__ uint8_t smem_raw[];
   __shared__ int s_abort;
   __shared__ float s_lse[kRowsPerCta];
+  __shared__ int s_par[kMaxNodes];
+  __shared__ uint64_t s_anc[kMaxNodes][2];
 
   pdl_launch_dependents();  // the LM head may start streaming its weights now
 
-  // The sequence extent and context length are caller inputs that the tree
-  // preparation kernel validates.  Before its verdict (pdl_wait below) this
-  // kernel only starts TMA copies of context K/V, whose coordinates stay
-  // inside the tensor maps whatever those inputs hold.
+  // This kernel does not depend on the tree preparation: it derives the
+  // ancestor masks itself and keeps every access inside the caller's arrays
+  // whatever the inputs hold (the preparation kernel reports malformed ones;
+  // the outputs of such a sequence are then unspecified).
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int rb = blockIdx.x, bg = blockIdx.y, z = blockIdx.z;
   const int b = bg / p.Hkv, g = bg - b * p.Hkv;
@@ -209,7 +233,10 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const __grid_constant__ 
   const int n = p.cu_nodes[b + 1] - s0;
   const int R = n * p.G;
   const int r0 = rb * kRowsPerCta;
-  if (n <= 0 || n > kMaxNodes || r0 >= R) return;
+  if (n <= 0 || n > kMaxNodes || s0 < 0 || s0 + n > p.T || r0 >= R) {
+    pdl_wait();
+    return;
+  }
   const int nrows = min(kRowsPerCta, R - r0);
   const KeyRange kr(z, p.split_len, min(p.ctx_len[b], p.ctx_max), n);
   const RowMap rm{s0, p.G, p.Hq, g, r0};
@@ -285,14 +312,6 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const __grid_constant__ 
     }
   }
 
-  pdl_wait();  // tree preparation results: sequence flags, ancestor masks
-  if (p.seq_flags[b] & (kSeqBadTree | kSeqBadCtx)) {
-    // skip the sequence, but only after the copies already started have landed
-    if (tid == 0)
-      for (int t = 0; t < kr.nctx && t < kAttnStages; ++t) mbar_wait(sBar + 8 * t, 0);
-    __syncthreads();
-    return;
-  }
   // after the tile loop the K stages hold this split's fp32 output rows
   float* s_o = reinterpret_cast<float*>(gK);
   if (kr.nctx + kr.ntree == 0) {
@@ -300,8 +319,10 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const __grid_constant__ 
     for (int r = tid; r < kRowsPerCta; r += 128) s_lse[r] = -INFINITY;
     for (int idx = tid; idx < kRowsPerCta * D; idx += 128) s_o[idx] = 0.f;
     cluster_merge<__nv_bfloat16, D>(p, rm, nrows, sK, smem_u32(s_lse));
+    pdl_wait();
     return;
   }
+  if (kr.ntree > 0) tree_ancestors(p.parent, s0, n, s_par, s_anc);
 
   // query rows -> shared memory (swizzled like the TMA tiles)
   const __nv_bfloat16* q = static_cast<const __nv_bfloat16*>(p.q);
@@ -327,14 +348,14 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const __grid_constant__ 
   uint64_t aAlo = 0, aAhi = 0, aBlo = 0, aBhi = 0;
   if (kr.ntree > 0) {
     if (rowA < nrows) {
-      const int node = s0 + (r0 + rowA) / p.G;
-      aAlo = p.anc[2 * node];
-      aAhi = p.anc[2 * node + 1];
+      const int node = (r0 + rowA) / p.G;
+      aAlo = s_anc[node][0];
+      aAhi = s_anc[node][1];
     }
     if (rowB < nrows) {
-      const int node = s0 + (r0 + rowB) / p.G;
-      aBlo = p.anc[2 * node];
-      aBhi = p.anc[2 * node + 1];
+      const int node = (r0 + rowB) / p.G;
+      aBlo = s_anc[node][0];
+      aBhi = s_anc[node][1];
     }
   }
 
@@ -490,6 +511,9 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const __grid_constant__ 
     s_lse[rowB] = (mB == -INFINITY) ? -INFINITY : mB * c + log2f(lB);
   }
   cluster_merge<__nv_bfloat16, D>(p, rm, nrows, sK, smem_u32(s_lse));
+  // complete only after the tree preparation has: the LM head's wait on this
+  // kernel then covers the preparation's outputs as well
+  pdl_wait();
 }
 
 // ----------------------------------------------------------- fp32 SIMT path
@@ -500,18 +524,21 @@ __global__ void __launch_bounds__(128) attn_f32_kernel(const AttnParams p) {
   constexpr int kPer = D / 32;
   extern __shared__ __align__(16) uint8_t smem_raw[];
   __shared__ float s_lse[kRowsPerCta];
+  __shared__ int s_par[kMaxNodes];
+  __shared__ uint64_t s_anc[kMaxNodes][2];
   float* s_o = reinterpret_cast<float*>(smem_raw);   // [64][D] split output rows
-  pdl_wait();
   pdl_launch_dependents();
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int rb = blockIdx.x, bg = blockIdx.y, z = blockIdx.z;
   const int b = bg / p.Hkv, g = bg - b * p.Hkv;
-  if (p.seq_flags[b] & (kSeqBadTree | kSeqBadCtx)) return;
   const int s0 = p.cu_nodes[b];
   const int n = p.cu_nodes[b + 1] - s0;
   const int R = n * p.G;
   const int r0 = rb * kRowsPerCta;
-  if (r0 >= R) return;
+  if (n <= 0 || n > kMaxNodes || s0 < 0 || s0 + n > p.T || r0 >= R) {
+    pdl_wait();
+    return;
+  }
   const int nrows = min(kRowsPerCta, R - r0);
   const KeyRange kr(z, p.split_len, min(p.ctx_len[b], p.ctx_max), n);
   const RowMap rm{s0, p.G, p.Hq, g, r0};
@@ -524,6 +551,7 @@ __global__ void __launch_bounds__(128) attn_f32_kernel(const AttnParams p) {
   const int ps = p.page_size;
   const int nctx_keys = max(0, kr.kend - kr.kbeg);
   const int ntree_keys = kr.ntree > 0 ? n : 0;
+  if (ntree_keys) tree_ancestors(p.parent, s0, n, s_par, s_anc);
 
   for (int r = warp; r < nrows; r += 4) {
     const size_t gr = rm.grow(r);
@@ -542,9 +570,9 @@ __global__ void __launch_bounds__(128) attn_f32_kernel(const AttnParams p) {
     }
     uint64_t alo = 0, ahi = 0;
     if (ntree_keys) {
-      const int node = s0 + (r0 + r) / p.G;
-      alo = p.anc[2 * node];
-      ahi = p.anc[2 * node + 1];
+      const int node = (r0 + r) / p.G;
+      alo = s_anc[node][0];
+      ahi = s_anc[node][1];
     }
     float m = -INFINITY, l = 0.f;
     for (int t = 0; t < nctx_keys + ntree_keys; ++t) {
@@ -591,6 +619,7 @@ __global__ void __launch_bounds__(128) attn_f32_kernel(const AttnParams p) {
     if (lane == 0) s_lse[r] = (m == -INFINITY) ? -INFINITY : m * c + log2f(l);
   }
   cluster_merge<float, D>(p, rm, nrows, smem_u32(s_o), smem_u32(s_lse));
+  pdl_wait();
 }
 
 }  // namespace

@@ -33,7 +33,6 @@ struct LmPartial {
 struct WsLayout {
   size_t status;       // int32[4]: [0] first device error code
   size_t seq_flags;    // int32[B]
-  size_t anc;          // uint64[T][2]: ancestor bitmask of each node (self included)
   size_t child_start;  // int32[T]: global slot of the node's first child
   size_t child_cnt;    // int32[T]
   size_t child_tok;    // int32[T]: children tokens, grouped by parent, sorted by (token, id)

@@ -37,7 +37,6 @@ struct PrepParams {
   const int32_t* ctx_len;   // may be null
   int* status;
   int* seq_flags;
-  uint64_t* anc;
   int32_t* child_start;
   int32_t* child_cnt;
   int32_t* child_tok;
@@ -57,8 +56,7 @@ struct AttnParams {
   const int32_t* cu_nodes;
   const int32_t* ctx_len;
   const int32_t* page_table;  // [B, ctx_max / ps] or null
-  const int* seq_flags;
-  const uint64_t* anc;
+  const int32_t* parent;      // local parent ids (ancestor masks are derived in-kernel)
   int* status;
   void* out;                // [T, Hq, D]
   int B, T, Hq, Hkv, G, D;
@@ -86,6 +84,8 @@ struct LmParams {
   float* l_draft;           // [T]
   int* status;
   int T, K, V, g_lm;
+  int a_rows;               // node rows per hidden-state TMA box: min(128, T rounded to 8);
+                            // A-tile rows past it are never loaded and never read
 };
 constexpr int kLmStages = 4;
 constexpr int kLmTileN = 256;      // vocabulary rows per MMA tile

@@ -178,7 +178,7 @@ __global__ void __launch_bounds__(192, 1)
           if (lane == 0) {
             const uint32_t a_s = base + stage * kStage;
             const uint32_t b_s = a_s + kATile;
-            mbar_expect_tx(full, static_cast<uint32_t>(kATile + nbox * kBoxBytes));
+            mbar_expect_tx(full, static_cast<uint32_t>(p.a_rows * 128 + nbox * kBoxBytes));
             tma_load_2d(a_s, &tm_h, full, kb * kKB, nt * kM, pol_h);
             for (int j = 0; j < nbox; ++j)
               tma_load_2d(b_s + j * kBoxBytes, &tm_w, full, kb * kKB, v0 + j * kLmBoxRows, pol_w);

@@ -1,7 +1,6 @@
-// Tree preparation: validates each draft tree and derives the structures the
-// attention and LM-head kernels consume.
-//  - ancestor bitmask of every node (self included): the tree part of the
-//    attention mask (a node sees its root-to-node path, Sec. 2 "Verify");
+// Tree preparation: validates each draft tree (parent array, drafted token
+// range, context length) into the status word and per-sequence flags, and
+// derives what the LM-head epilogue consumes:
 //  - children of every node grouped by parent and sorted by (token, node id),
 //    so the LM-head epilogue can pick l_draft = logits[parent, token] while it
 //    sweeps the vocabulary in increasing order (Eq. 1 needs the parent row's
@@ -63,18 +62,6 @@ __global__ void __launch_bounds__(kMaxNodes) tree_prep_kernel(PrepParams p) {
   const bool tree_ok = !(bad & kSeqBadTree);
 
   if (i < n) {
-    // ancestors: walk up the (validated, strictly decreasing) parent chain
-    uint64_t a0 = 0, a1 = 0;
-    int u = i;
-    while (u >= 0) {
-      if (u < 64)
-        a0 |= 1ull << u;
-      else
-        a1 |= 1ull << (u - 64);
-      u = tree_ok ? s_par[u] : -1;
-    }
-    p.anc[2 * (s + i)] = a0;
-    p.anc[2 * (s + i) + 1] = a1;
     int c = 0;
     if (tree_ok)
       for (int j = 1; j < n; ++j) c += (s_par[j] == i);
