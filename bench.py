@@ -128,6 +128,23 @@ class Clocks:
                 "sm_max_mhz": max(mx) if mx else None, "reasons": reasons, "samples": len(rows)}
 
 
+def slowest_rank(values, world, device):
+    """Element-wise maximum of per-rank timings over all ranks (the job is as
+    fast as its slowest replica)."""
+    if world == 1:
+        return list(values)
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor(values, dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return [float(x) for x in t]
+
+
+def job_value(nodes_per_rank, world, seconds):
+    """Whole-job throughput: every rank verifies its own replica (weak scaling)."""
+    return world * nodes_per_rank / seconds
+
+
 def ranks_torch(wl, device):
     """Top-5 tokens of every parent row, for the drafted-token mixture (input
     synthesis with a torch fp32 matmul on the device, outside any timing)."""
@@ -311,10 +328,7 @@ def run_asd(args):
     stage_ms = stage.mean(axis=0)
     staged_ms = float(np.mean([evs[k][0].elapsed_time(evs[k][4]) for k in range(K)]))
     lm_ms = float(stage_ms[2])
-    if world > 1:
-        t = torch.tensor([ms, lm_ms], device=device, dtype=torch.float64)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms, lm_ms_max = float(t[0]), float(t[1])
+    ms, lm_ms = slowest_rank([ms, lm_ms], world, device)
     mean_path = float(step.out["path_len"].float().mean())
 
     # end to end through the public API: per step, H2D of the step's inputs
@@ -346,11 +360,8 @@ def run_asd(args):
                 v.copy_(step.out[k2], non_blocking=True)
             stream.synchronize()
         e2e_s = (time.perf_counter() - t0) / K
-        if world > 1:
-            t = torch.tensor([e2e_s], device=device, dtype=torch.float64)
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            e2e_s = float(t[0])
-        e2e = {"value": world * wl.T / e2e_s, "unit": UNIT, "h2d_bytes_per_step": h2d,
+        (e2e_s,) = slowest_rank([e2e_s], world, device)
+        e2e = {"value": job_value(wl.T, world, e2e_s), "unit": UNIT, "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": d2h, "us_per_step": 1e6 * e2e_s}
 
     if rank != 0:
@@ -362,7 +373,7 @@ def run_asd(args):
     achieved = lmb / (lm_ms * 1e-3) / 1e9
     sb = step_bytes(wl, mean_path)
     line = {
-        "metric": METRIC, "value": world * wl.T / (ms * 1e-3), "unit": UNIT, "n_gpus": world,
+        "metric": METRIC, "value": job_value(wl.T, world, ms * 1e-3), "unit": UNIT, "n_gpus": world,
         "steps": K, "warmup": W, "ms_per_step": ms, "us_per_step": 1e3 * ms,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic (seeded; Llama-3.1-8B-shaped tensors, random weights)",
