@@ -34,6 +34,10 @@ UNIT = "nodes/s"
 CONFIG = 2
 TAU = 0.3
 N_STAGE_KERNELS = 4   # prep, attention (splits merged in-kernel), LM head, tail
+# DRAM bytes (read + write) of one LM-head launch on this workload, from the
+# ncu capture summarised in profiles/verify_step_llama8b_b1_ctx2048_tree60.md;
+# set to None whenever lmhead_tc.cu changes until it is captured again.
+LMHEAD_TRAFFIC_BYTES = 1054184000
 
 
 def parse():
@@ -383,7 +387,7 @@ def run_asd(args):
                      "peak": peak, "unit": "GB/s", "frac": achieved / peak,
                      "peak_source": peak_kind + " hbm_gbs (MEASURED_PEAKS.json)",
                      "algorithmic_bytes_per_launch": lmb, "avg_launch_us": 1e3 * lm_ms,
-                     "traffic": None},
+                     "traffic": LMHEAD_TRAFFIC_BYTES},
         "stages_us": {"prep": 1e3 * stage_ms[0], "attention": 1e3 * stage_ms[1],
                       "lmhead": 1e3 * stage_ms[2], "tail": 1e3 * stage_ms[3],
                       "step_with_stage_events": 1e3 * staged_ms,
