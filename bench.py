@@ -33,11 +33,12 @@ METRIC = "verified tree nodes/s"
 UNIT = "nodes/s"
 CONFIG = 2
 TAU = 0.3
-N_STAGE_KERNELS = 4   # prep, attention (splits merged in-kernel), LM head, tail
+N_STAGE_KERNELS = 4   # prep, LM head, attention (splits merged in-kernel), tail
+STAGES = ("prep", "lmhead", "attention", "tail")   # order of the stage events
 # DRAM bytes (read + write) of one LM-head launch on this workload, from the
 # ncu capture summarised in profiles/verify_step_llama8b_b1_ctx2048_tree60.md;
 # set to None whenever lmhead_tc.cu changes until it is captured again.
-LMHEAD_TRAFFIC_BYTES = 1054184000
+LMHEAD_TRAFFIC_BYTES = None
 
 
 def parse():
@@ -331,7 +332,7 @@ def run_asd(args):
     stage = np.array([[evs[k][j].elapsed_time(evs[k][j + 1]) for j in range(4)] for k in range(K)])
     stage_ms = stage.mean(axis=0)
     staged_ms = float(np.mean([evs[k][0].elapsed_time(evs[k][4]) for k in range(K)]))
-    lm_ms = float(stage_ms[2])
+    lm_ms = float(stage_ms[STAGES.index("lmhead")])
     ms, lm_ms = slowest_rank([ms, lm_ms], world, device)
     mean_path = float(step.out["path_len"].float().mean())
 
@@ -388,8 +389,7 @@ def run_asd(args):
                      "peak_source": peak_kind + " hbm_gbs (MEASURED_PEAKS.json)",
                      "algorithmic_bytes_per_launch": lmb, "avg_launch_us": 1e3 * lm_ms,
                      "traffic": LMHEAD_TRAFFIC_BYTES},
-        "stages_us": {"prep": 1e3 * stage_ms[0], "attention": 1e3 * stage_ms[1],
-                      "lmhead": 1e3 * stage_ms[2], "tail": 1e3 * stage_ms[3],
+        "stages_us": {**{name: 1e3 * stage_ms[j] for j, name in enumerate(STAGES)},
                       "step_with_stage_events": 1e3 * staged_ms,
                       "note": "second timed region with events between kernels (no overlap)"},
         "mean_path_len": mean_path,

@@ -205,8 +205,9 @@ typedef struct asd_verify_args {
   int32_t* n_promoted;
   int32_t* ctx_len_out;
   /* optional cudaEvent_t handles (NULL to skip), recorded on `stream` at:
-     [0] start, [1] after tree preparation, [2] after attention,
-     [3] after the LM-head GEMM kernel, [4] after path choice and commit. */
+     [0] start, [1] after tree preparation, [2] after the LM-head GEMM
+     kernel, [3] after attention, [4] after path choice and commit.  An event
+     between two kernels stops them from overlapping. */
   void* stage_events[ASD_NUM_STAGE_EVENTS];
 } asd_verify_args;
 

@@ -90,14 +90,14 @@ WsLayout layout(const asd_dims& d, int T, int nsm) {
   WsLayout L{};
   const int G = d.num_q_heads / d.num_kv_heads;
   L.g_lm = std::max(1, std::min(std::min(nsm, kMaxLmRanges), (d.vocab + kLmBoxRows - 1) / kLmBoxRows));
-  // context splits: enough CTAs for about one wave at two CTAs per SM, at
-  // most kMaxAttnParts (the splits of a row block form one thread-block
-  // cluster); the last non-empty split of a sequence also takes its tree keys
+  // context splits: at most one attention CTA per SM (in a verify step each
+  // shares its SM with an LM-head CTA), at most kMaxAttnParts (the splits of a
+  // row block form one thread-block cluster); the last non-empty split of a
+  // sequence also takes its tree keys
   const int rblocks = attention_row_blocks(d.max_nodes, G);
   const long long base = static_cast<long long>(rblocks) * d.batch * d.num_kv_heads;
-  const long long target = 2LL * nsm;
   const int max_splits = std::max(1, std::min(kMaxAttnParts, (d.ctx_max + 63) / 64));
-  long long ns = (target + base - 1) / base;
+  long long ns = nsm / base;
   ns = std::max(1LL, std::min(ns, static_cast<long long>(max_splits)));
   const int per = static_cast<int>((std::max(d.ctx_max, 1) + ns - 1) / ns);
   L.split_len = ((per + 63) / 64) * 64;
@@ -211,10 +211,10 @@ asd_status run_attention(const Ctx& c, const void* q, const void* k_cache, const
     uint32_t box_rows;
     if (d.page_size == 0) {
       rows = static_cast<uint64_t>(d.batch) * d.num_kv_heads * static_cast<uint64_t>(d.ctx_max);
-      box_rows = 64;
+      box_rows = static_cast<uint32_t>(attention_keys_per_tile());
     } else {
       rows = static_cast<uint64_t>(d.num_pages) * d.num_kv_heads * d.page_size;
-      box_rows = d.page_size < 64 ? d.page_size : 64;
+      box_rows = static_cast<uint32_t>(std::min(d.page_size, attention_keys_per_tile()));
     }
     if (rows == 0) rows = 1;  // no context at all: the map is never used
     if (!make_tmap_bf16(&tk, k_cache, d.head_dim, rows, box_rows) ||
@@ -447,11 +447,14 @@ asd_status asd_verify_step(const asd_dims* dims, const asd_verify_args* a, void*
                        c.st) != cudaSuccess)
     return ASD_ERR_CUDA;
   record(a->stage_events[1], c.st);
-  st = run_attention(c, a->q, a->k_cache, a->v_cache, a->page_table, a->ctx_len, a->tree_k,
-                     a->tree_v, a->parent, a->cu_nodes, a->attn_out);
+  // The LM head goes first and takes one CTA per SM; the attention kernel
+  // starts right behind it (it reads no output of the LM head) and its CTAs
+  // share the SMs with the LM head's while the weights stream in.
+  st = run_lmhead(c, a->hidden, a->w_lm, a->l_draft);
   if (st != ASD_OK) return st;
   record(a->stage_events[2], c.st);
-  st = run_lmhead(c, a->hidden, a->w_lm, a->l_draft);
+  st = run_attention(c, a->q, a->k_cache, a->v_cache, a->page_table, a->ctx_len, a->tree_k,
+                     a->tree_v, a->parent, a->cu_nodes, a->attn_out);
   if (st != ASD_OK) return st;
   record(a->stage_events[3], c.st);
   TailParams t = tail_params(c, kTailFinalize | kTailWalk | kTailCompact);

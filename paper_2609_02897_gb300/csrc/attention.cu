@@ -7,7 +7,7 @@
 // row r -> node r / G, head g*G + r % G.  Split z covers context keys
 // [z*L, (z+1)*L) (flash-decoding split-KV); the CTA of the sequence's last
 // non-empty split also covers the tree keys, where a node only sees its
-// ancestors (bitmask from the tree preparation kernel).  The splits of one
+// ancestors (bitmasks derived in-kernel from the parent array).  The splits of one
 // (row block, sequence x KV head) form a thread-block cluster: each CTA keeps
 // its softmax-normalised partial output and log-sum-exp in shared memory, and
 // after a cluster barrier every CTA merges a slice of the rows by reading its
@@ -19,8 +19,10 @@ namespace asd {
 namespace {
 
 constexpr int kRowsPerCta = 64;   // 4 warps x 16 query rows
-constexpr int kKeysPerTile = 64;
-constexpr int kAttnStages = 2;    // 2 CTAs per SM fit with D = 128
+constexpr int kKeysPerTile = 32;  // keys per K/V tile (TMA box rows)
+constexpr int kAttnStages = 2;
+// With D = 128 a CTA takes 1 KB + 16 KB (Q) + 32 KB (K/V ring) of dynamic
+// shared memory, small enough to share an SM with an LM-head CTA.
 
 // ---------------------------------------------------------------- mma helpers
 __device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
@@ -54,9 +56,11 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
 }
 
 // Tile layout in shared memory (the TMA 128-byte swizzle): [D/64 halves]
-// [64 rows][128 bytes]; 16-byte chunk c of row r sits at chunk c ^ (r & 7).
+// [ROWS rows][128 bytes]; 16-byte chunk c of row r sits at chunk c ^ (r & 7).
+template <int ROWS>
 __device__ __forceinline__ uint32_t sw_off(int row, int chunk) {
-  return static_cast<uint32_t>((chunk >> 3) * 8192 + row * 128 + (((chunk & 7) ^ (row & 7)) << 4));
+  return static_cast<uint32_t>((chunk >> 3) * (ROWS * 128) + row * 128 +
+                               (((chunk & 7) ^ (row & 7)) << 4));
 }
 
 __device__ __forceinline__ bool anc_bit(uint64_t lo, uint64_t hi, int j) {
@@ -211,16 +215,21 @@ template <int D>
 __global__ void __launch_bounds__(128) attn_bf16_kernel(const __grid_constant__ CUtensorMap tm_k,
                                                         const __grid_constant__ CUtensorMap tm_v,
                                                         const AttnParams p) {
-  constexpr int kTileBytes = kKeysPerTile * D * 2;
+  constexpr int kTileBytes = kKeysPerTile * D * 2;   // one K or V tile
+  constexpr int kQBytes = kRowsPerCta * D * 2;
+  constexpr int kHalf = kKeysPerTile * 128;           // one 64-column half of a tile
   constexpr int kNH = D / 64;
   constexpr int kChunks = D / 8;
+  constexpr int kNT = kKeysPerTile / 8;               // 8-key n-tiles of S per tile
+  static_assert(2 * kAttnStages * kTileBytes >= kRowsPerCta * D * 4,
+                "the K/V ring must hold the fp32 output rows");
   extern __shared__ uint8_t smem_raw[];
   __shared__ int s_abort;
   __shared__ float s_lse[kRowsPerCta];
   __shared__ int s_par[kMaxNodes];
   __shared__ uint64_t s_anc[kMaxNodes][2];
 
-  pdl_launch_dependents();  // the LM head may start streaming its weights now
+  pdl_launch_dependents();  // nothing downstream reads this kernel's output early
 
   // This kernel does not depend on the tree preparation: it derives the
   // ancestor masks itself and keeps every access inside the caller's arrays
@@ -246,11 +255,11 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const __grid_constant__ 
   uint8_t* smem = smem_raw + pad;
   base += pad;
   const uint32_t sQ = base;
-  const uint32_t sK = sQ + kTileBytes;
+  const uint32_t sK = sQ + kQBytes;
   const uint32_t sV = sK + kAttnStages * kTileBytes;
   const uint32_t sBar = sV + kAttnStages * kTileBytes;
   uint8_t* gQ = smem;
-  uint8_t* gK = smem + kTileBytes;
+  uint8_t* gK = smem + kQBytes;
   uint8_t* gV = gK + kAttnStages * kTileBytes;
 
   const int ps = p.page_size;
@@ -266,13 +275,13 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const __grid_constant__ 
       mbar_expect_tx(bar, 2 * kTileBytes);
 #pragma unroll
       for (int h = 0; h < kNH; ++h) {
-        tma_load_2d(dK + h * 8192, &tm_k, bar, h * 64, row, pol);
-        tma_load_2d(dV + h * 8192, &tm_v, bar, h * 64, row, pol);
+        tma_load_2d(dK + h * kHalf, &tm_k, bar, h * 64, row, pol);
+        tma_load_2d(dV + h * kHalf, &tm_v, bar, h * 64, row, pol);
       }
     } else {
-      const int br = ps < 64 ? ps : 64;  // rows per box
+      const int br = ps < kKeysPerTile ? ps : kKeysPerTile;  // rows per box
       const int nbox = kKeysPerTile / br;
-      int rows[kKeysPerTile / 8];        // at most 8 boxes (page_size >= 8)
+      int rows[kKeysPerTile / 8];        // page_size >= 8
       int cnt = 0;
       for (int j = 0; j < nbox; ++j) {
         const int key = key0 + j * br;
@@ -291,8 +300,8 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const __grid_constant__ 
         if (rows[j] < 0) continue;
 #pragma unroll
         for (int h = 0; h < kNH; ++h) {
-          tma_load_2d(dK + h * 8192 + j * br * 128, &tm_k, bar, h * 64, rows[j], pol);
-          tma_load_2d(dV + h * 8192 + j * br * 128, &tm_v, bar, h * 64, rows[j], pol);
+          tma_load_2d(dK + h * kHalf + j * br * 128, &tm_k, bar, h * 64, rows[j], pol);
+          tma_load_2d(dV + h * kHalf + j * br * 128, &tm_v, bar, h * 64, rows[j], pol);
         }
       }
     }
@@ -312,7 +321,7 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const __grid_constant__ 
     }
   }
 
-  // after the tile loop the K stages hold this split's fp32 output rows
+  // after the tile loop the K/V ring holds this split's fp32 output rows
   float* s_o = reinterpret_cast<float*>(gK);
   if (kr.nctx + kr.ntree == 0) {
     // empty split: weight-zero log-sum-exp and finite (zero) rows for the merge
@@ -330,7 +339,7 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const __grid_constant__ 
     const int r = c / kChunks, ch = c - r * kChunks;
     uint4 v = make_uint4(0u, 0u, 0u, 0u);
     if (r < nrows) v = *reinterpret_cast<const uint4*>(q + rm.grow(r) * D + ch * 8);
-    *reinterpret_cast<uint4*>(gQ + sw_off(r, ch)) = v;
+    *reinterpret_cast<uint4*>(gQ + sw_off<kRowsPerCta>(r, ch)) = v;
   }
   __syncthreads();
 
@@ -340,7 +349,7 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const __grid_constant__ 
   for (int ks = 0; ks < D / 16; ++ks) {
     const int row = warp * 16 + (lane & 7) + (((lane >> 3) & 1) << 3);
     const int chunk = 2 * ks + (lane >> 4);
-    ldsm_x4(sQ + sw_off(row, chunk), qa[ks][0], qa[ks][1], qa[ks][2], qa[ks][3]);
+    ldsm_x4(sQ + sw_off<kRowsPerCta>(row, chunk), qa[ks][0], qa[ks][1], qa[ks][2], qa[ks][3]);
   }
 
   // ancestor masks of this thread's two rows (tree tiles only)
@@ -385,8 +394,8 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const __grid_constant__ 
           kv = *reinterpret_cast<const uint4*>(tk + off);
           vv = *reinterpret_cast<const uint4*>(tv + off);
         }
-        *reinterpret_cast<uint4*>(gKs + sw_off(r, ch)) = kv;
-        *reinterpret_cast<uint4*>(gVs + sw_off(r, ch)) = vv;
+        *reinterpret_cast<uint4*>(gKs + sw_off<kKeysPerTile>(r, ch)) = kv;
+        *reinterpret_cast<uint4*>(gVs + sw_off<kKeysPerTile>(r, ch)) = vv;
       }
     } else {
       const bool ok = mbar_wait(sBar + 8 * stage, (t / kAttnStages) & 1);
@@ -397,7 +406,7 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const __grid_constant__ 
         // rows past the context may hold anything: zero V so that 0 * V stays 0
         for (int cidx = tid; cidx < (kKeysPerTile - valid) * kChunks; cidx += 128) {
           const int r = valid + cidx / kChunks, ch = cidx % kChunks;
-          *reinterpret_cast<uint4*>(gVs + sw_off(r, ch)) = make_uint4(0u, 0u, 0u, 0u);
+          *reinterpret_cast<uint4*>(gVs + sw_off<kKeysPerTile>(r, ch)) = make_uint4(0u, 0u, 0u, 0u);
         }
       }
     }
@@ -405,17 +414,17 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const __grid_constant__ 
     if (s_abort) break;
 
     const uint32_t aK = sK + stage * kTileBytes, aV = sV + stage * kTileBytes;
-    float sc[8][4];
+    float sc[kNT][4];
 #pragma unroll
-    for (int j = 0; j < 8; ++j) sc[j][0] = sc[j][1] = sc[j][2] = sc[j][3] = 0.f;
+    for (int j = 0; j < kNT; ++j) sc[j][0] = sc[j][1] = sc[j][2] = sc[j][3] = 0.f;
 #pragma unroll
     for (int ks = 0; ks < D / 16; ++ks) {
 #pragma unroll
-      for (int nj = 0; nj < 4; ++nj) {
+      for (int nj = 0; nj < kNT / 2; ++nj) {
         uint32_t b0, b1, b2, b3;
         const int key = 16 * nj + (lane & 7) + ((lane >> 4) << 3);
         const int chunk = 2 * ks + ((lane >> 3) & 1);
-        ldsm_x4(aK + sw_off(key, chunk), b0, b1, b2, b3);
+        ldsm_x4(aK + sw_off<kKeysPerTile>(key, chunk), b0, b1, b2, b3);
         mma_bf16(sc[2 * nj], qa[ks], b0, b1);
         mma_bf16(sc[2 * nj + 1], qa[ks], b2, b3);
       }
@@ -423,7 +432,7 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const __grid_constant__ 
     // mask and online softmax (scores in raw units; exp2 with the folded scale)
     float mxA = -INFINITY, mxB = -INFINITY;
 #pragma unroll
-    for (int j = 0; j < 8; ++j) {
+    for (int j = 0; j < kNT; ++j) {
 #pragma unroll
       for (int e = 0; e < 2; ++e) {
         const int local = 8 * j + 2 * kq + e;
@@ -459,7 +468,7 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const __grid_constant__ 
     }
     const float nA = -muA * c, nB = -muB * c;
 #pragma unroll
-    for (int j = 0; j < 8; ++j) {
+    for (int j = 0; j < kNT; ++j) {
       sc[j][0] = exp2f(fmaf(sc[j][0], c, nA));
       sc[j][1] = exp2f(fmaf(sc[j][1], c, nA));
       sc[j][2] = exp2f(fmaf(sc[j][2], c, nB));
@@ -469,7 +478,7 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const __grid_constant__ 
     }
     // O += P V
 #pragma unroll
-    for (int kk = 0; kk < 4; ++kk) {
+    for (int kk = 0; kk < kKeysPerTile / 16; ++kk) {
       uint32_t pa[4];
       pa[0] = pack_bf16(sc[2 * kk][0], sc[2 * kk][1]);
       pa[1] = pack_bf16(sc[2 * kk][2], sc[2 * kk][3]);
@@ -480,7 +489,7 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const __grid_constant__ 
         uint32_t b0, b1, b2, b3;
         const int key = 16 * kk + (lane & 7) + (((lane >> 3) & 1) << 3);
         const int chunk = 2 * dp + (lane >> 4);
-        ldsm_x4_t(aV + sw_off(key, chunk), b0, b1, b2, b3);
+        ldsm_x4_t(aV + sw_off<kKeysPerTile>(key, chunk), b0, b1, b2, b3);
         mma_bf16(o[2 * dp], pa, b0, b1);
         mma_bf16(o[2 * dp + 1], pa, b2, b3);
       }
@@ -511,8 +520,8 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const __grid_constant__ 
     s_lse[rowB] = (mB == -INFINITY) ? -INFINITY : mB * c + log2f(lB);
   }
   cluster_merge<__nv_bfloat16, D>(p, rm, nrows, sK, smem_u32(s_lse));
-  // complete only after the tree preparation has: the LM head's wait on this
-  // kernel then covers the preparation's outputs as well
+  // complete only after the previous kernel in the stream has: a later
+  // kernel's wait on this one then covers that kernel's outputs as well
   pdl_wait();
 }
 
@@ -626,8 +635,11 @@ __global__ void __launch_bounds__(128) attn_f32_kernel(const AttnParams p) {
 
 size_t attn_bf16_smem_bytes(int D) {
   const size_t tile = static_cast<size_t>(kKeysPerTile) * D * 2;
-  return 1024 + tile * (1 + 2 * kAttnStages) + 8 * kAttnStages;
+  const size_t q = static_cast<size_t>(kRowsPerCta) * D * 2;
+  return 1024 + q + tile * 2 * kAttnStages + 8 * kAttnStages;
 }
+
+int attention_keys_per_tile() { return kKeysPerTile; }
 
 int attention_row_blocks(int max_nodes, int G) {
   return (max_nodes * G + kRowsPerCta - 1) / kRowsPerCta;
@@ -662,15 +674,11 @@ cudaError_t launch_attention_bf16(const AttnParams& p, const CUtensorMap& tm_k,
                                   const CUtensorMap& tm_v, cudaStream_t s) {
   const size_t smem = attn_bf16_smem_bytes(p.D);
   if (p.D == 128) {
-    cudaError_t err = cudaFuncSetAttribute(attn_bf16_kernel<128>,
-                                           cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                           static_cast<int>(smem));
+    cudaError_t err = set_smem_attrs(attn_bf16_kernel<128>, smem);
     if (err != cudaSuccess) return err;
     return launch_attn(attn_bf16_kernel<128>, p, smem, s, tm_k, tm_v, p);
   }
-  cudaError_t err = cudaFuncSetAttribute(attn_bf16_kernel<64>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(smem));
+  cudaError_t err = set_smem_attrs(attn_bf16_kernel<64>, smem);
   if (err != cudaSuccess) return err;
   return launch_attn(attn_bf16_kernel<64>, p, smem, s, tm_k, tm_v, p);
 }

@@ -29,6 +29,18 @@ cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t s
   return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
 }
 
+// Dynamic shared memory limit of `kernel`, and the whole unified L1 as shared
+// memory, so that an LM-head CTA and an attention CTA fit on one SM together
+// (the default carveout is sized for one kernel's CTAs alone).
+template <typename K>
+cudaError_t set_smem_attrs(K* kernel, size_t smem) {
+  cudaError_t err = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(smem));
+  if (err != cudaSuccess) return err;
+  return cudaFuncSetAttribute(kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
+                              cudaSharedmemCarveoutMaxShared);
+}
+
 // ------------------------------------------------------------ tree preparation
 struct PrepParams {
   const int32_t* parent;
@@ -65,12 +77,14 @@ struct AttnParams {
   float scale_log2;         // log2(e) / sqrt(D)
 };
 // bf16 path: tensor-core (mma.sync) split-KV kernel fed by TMA; tm_k / tm_v are
-// 2D tensor maps over the context cache rows (box 64 x min(64, rows per page)).
+// 2D tensor maps over the context cache rows (box 64 columns x
+// min(attention_keys_per_tile(), rows per page) rows).
 // Both paths merge the splits of a group inside its thread-block cluster.
 cudaError_t launch_attention_bf16(const AttnParams& p, const CUtensorMap& tm_k,
                                   const CUtensorMap& tm_v, cudaStream_t s);
 cudaError_t launch_attention_f32(const AttnParams& p, cudaStream_t s);
 int attention_row_blocks(int max_nodes, int G);
+int attention_keys_per_tile();   // context keys per K/V tile = TMA box rows
 
 // -------------------------------------------------------------------- LM head
 struct LmParams {
@@ -87,7 +101,7 @@ struct LmParams {
   int a_rows;               // node rows per hidden-state TMA box: min(128, T rounded to 8);
                             // A-tile rows past it are never loaded and never read
 };
-constexpr int kLmStages = 4;
+constexpr int kLmStages = 3;      // 3 x 48 KB: leaves room for an attention CTA on the SM
 constexpr int kLmTileN = 256;      // vocabulary rows per MMA tile
 constexpr int kLmBoxRows = 32;     // vocabulary rows per TMA box
 size_t lmhead_tc_smem_bytes();

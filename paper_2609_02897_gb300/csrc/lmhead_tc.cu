@@ -313,9 +313,7 @@ size_t lmhead_tc_smem_bytes() { return 1024 + static_cast<size_t>(kLmStages) * k
 cudaError_t launch_lmhead_bf16(const LmParams& p, const CUtensorMap& tm_hidden,
                                const CUtensorMap& tm_w, cudaStream_t s) {
   const size_t smem = lmhead_tc_smem_bytes();
-  cudaError_t err = cudaFuncSetAttribute(lmhead_tc_kernel,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(smem));
+  cudaError_t err = set_smem_attrs(lmhead_tc_kernel, smem);
   if (err != cudaSuccess) return err;
   return launch_pdl(lmhead_tc_kernel, dim3(p.g_lm), dim3(192), smem, s, tm_hidden, tm_w, p);
 }
