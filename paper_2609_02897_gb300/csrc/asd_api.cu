@@ -246,11 +246,12 @@ asd_status run_lmhead(const Ctx& c, const void* hidden, const void* w, float* l_
   p.a_rows = std::min(128, (c.T + 7) / 8 * 8);
   cudaError_t err;
   if (d.dtype == ASD_BF16) {
-    CUtensorMap th, tw;
+    CUtensorMap th, tw64, tw32;
     if (!make_tmap_bf16(&th, hidden, d.hidden, c.T, static_cast<uint32_t>(p.a_rows)) ||
-        !make_tmap_bf16(&tw, w, d.hidden, d.vocab, kLmBoxRows))
+        !make_tmap_bf16(&tw64, w, d.hidden, d.vocab, 2 * kLmBoxRows) ||
+        !make_tmap_bf16(&tw32, w, d.hidden, d.vocab, kLmBoxRows))
       return ASD_ERR_CUDA;
-    err = launch_lmhead_bf16(p, th, tw, c.st);
+    err = launch_lmhead_bf16(p, th, tw64, tw32, c.st);
   } else {
     err = launch_lmhead_f32(p, c.st);
   }

@@ -99,15 +99,17 @@ struct LmParams {
   int* status;
   int T, K, V, g_lm;
   int a_rows;               // node rows per hidden-state TMA box: min(128, T rounded to 8);
-                            // A-tile rows past it are never loaded and never read
+                            // accumulator rows past it belong to no node
 };
-constexpr int kLmStages = 3;      // 3 x 48 KB: leaves room for an attention CTA on the SM
-constexpr int kLmTileN = 256;      // vocabulary rows per MMA tile
-constexpr int kLmBoxRows = 32;     // vocabulary rows per TMA box
-size_t lmhead_tc_smem_bytes();
+constexpr int kLmStages = 3;       // 3 x 48 KB (a_rows <= 64): room for an attention CTA
+constexpr int kLmTileN = 128;      // vocabulary rows per MMA tile
+constexpr int kLmBoxRows = 32;     // vocabulary rows per range group (and per small TMA box)
+size_t lmhead_tc_smem_bytes(int a_rows);
 // bf16 path: tcgen05/TMEM GEMM with the fused max/argmax/sum-exp/l_draft epilogue.
+// tm_w64 / tm_w32: tensor maps over W [V, K] with boxes of 64 and 32 rows.
 cudaError_t launch_lmhead_bf16(const LmParams& p, const CUtensorMap& tm_hidden,
-                               const CUtensorMap& tm_w, cudaStream_t s);
+                               const CUtensorMap& tm_w64, const CUtensorMap& tm_w32,
+                               cudaStream_t s);
 cudaError_t launch_lmhead_f32(const LmParams& p, cudaStream_t s);
 
 // --------------------------------------- finalize / accepted path / K/V commit

@@ -8,8 +8,14 @@
 // running max, lowest argmax, sum of exp and the drafted tokens' logits.
 // Logits never leave the SM.  Each CTA owns one contiguous vocabulary range
 // (one CTA per SM, ranges balanced to 32 rows), streams its slice of W once
-// per 128-node tile through a 4-stage TMA ring, and writes one partial
+// per 128-node tile through a 3-stage TMA ring, and writes one partial
 // (max, argmax, sum-exp) per node; the tail kernel merges the ranges.
+//
+// A stage holds two k-blocks (128 hidden elements) of a 128-row vocabulary
+// tile (W, 32 KB, in 64-row TMA boxes) and of the node tile (hidden states,
+// a_rows rows).  Reading 256 contiguous bytes of each weight row per stage,
+// in few large boxes, streams W from HBM markedly faster than one k-block of
+// a 256-row tile per stage.
 //
 // Warp roles (192 threads): warp 0 TMA producer, warp 1 TMEM allocator and
 // MMA issuer, warps 2-5 epilogue (TMEM lane quarters 2, 3, 0, 1).
@@ -21,11 +27,19 @@ namespace {
 
 constexpr int kM = 128;                        // node rows per MMA = TMEM lanes
 constexpr int kKB = 64;                        // hidden elements per k-block (128 B)
-constexpr int kATile = kM * 128;               // 16 KB
-constexpr int kBTile = kLmTileN * 128;         // 32 KB
-constexpr int kStage = kATile + kBTile;
-constexpr int kBoxBytes = kLmBoxRows * 128;    // 4 KB
+constexpr int kKbPerStage = 2;
+constexpr int kBTile = kLmTileN * 128;         // W rows of one k-block: 16 KB
+constexpr int kGroupBytes = kLmBoxRows * 128;  // one 32-row group of one k-block: 4 KB
 constexpr uint32_t kTmemCols = 2 * kLmTileN;   // two accumulators
+
+// Stage slot: the node rows of both k-blocks (a_rows x 128 B each), then W.
+// The MMA reads 128 A rows from each k-block's start; rows past a_rows fall
+// on the next block of the same slot and only feed accumulator rows that
+// no node owns.
+__host__ __device__ constexpr int lm_a_bytes(int a_rows) { return kKbPerStage * a_rows * 128; }
+__host__ __device__ constexpr int lm_slot_bytes(int a_rows) {
+  return lm_a_bytes(a_rows) + kKbPerStage * kBTile;
+}
 
 __device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
   uint64_t d = static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);  // start address >> 4
@@ -104,7 +118,8 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
 
 __global__ void __launch_bounds__(192, 1)
     lmhead_tc_kernel(const __grid_constant__ CUtensorMap tm_h,
-                     const __grid_constant__ CUtensorMap tm_w, const LmParams p) {
+                     const __grid_constant__ CUtensorMap tm_w64,
+                     const __grid_constant__ CUtensorMap tm_w32, const LmParams p) {
   extern __shared__ uint8_t smem_raw[];
   __shared__ __align__(8) uint64_t s_full[kLmStages];
   __shared__ __align__(8) uint64_t s_empty[kLmStages];
@@ -127,6 +142,9 @@ __global__ void __launch_bounds__(192, 1)
   const int nvt = ve > vs ? (ve - vs + kLmTileN - 1) / kLmTileN : 0;
   const int nnt = (p.T + kM - 1) / kM;
   const int nkb = (p.K + kKB - 1) / kKB;
+  const int nkp = (nkb + kKbPerStage - 1) / kKbPerStage;   // stages per tile
+  const int a_blk = p.a_rows * 128;                         // one k-block of node rows
+  const int slot = lm_slot_bytes(p.a_rows);
 
   uint32_t base = smem_u32(smem_raw);
   base += (1024u - (base & 1023u)) & 1023u;
@@ -157,7 +175,8 @@ __global__ void __launch_bounds__(192, 1)
     uint64_t pol_w = 0, pol_h = 0;
     if (lane == 0) {
       prefetch_tmap(&tm_h);
-      prefetch_tmap(&tm_w);
+      prefetch_tmap(&tm_w64);
+      prefetch_tmap(&tm_w32);
       pol_w = l2_policy_evict_first();
       pol_h = l2_policy_evict_last();
     }
@@ -167,8 +186,8 @@ __global__ void __launch_bounds__(192, 1)
     for (int nt = 0; nt < nnt && ok; ++nt) {
       for (int vt = 0; vt < nvt && ok; ++vt) {
         const int v0 = vs + vt * kLmTileN;
-        const int nbox = (min(kLmTileN, ve - v0) + kLmBoxRows - 1) / kLmBoxRows;
-        for (int kb = 0; kb < nkb; ++kb) {
+        const int ng = (min(kLmTileN, ve - v0) + kLmBoxRows - 1) / kLmBoxRows;  // 32-row groups
+        for (int kp = 0; kp < nkp; ++kp) {
           const uint32_t full = smem_u32(&s_full[stage]);
           ok = __shfl_sync(0xffffffffu, mbar_wait(smem_u32(&s_empty[stage]), ph ^ 1u), 0);
           if (!ok || s_abort) {
@@ -176,12 +195,21 @@ __global__ void __launch_bounds__(192, 1)
             break;
           }
           if (lane == 0) {
-            const uint32_t a_s = base + stage * kStage;
-            const uint32_t b_s = a_s + kATile;
-            mbar_expect_tx(full, static_cast<uint32_t>(p.a_rows * 128 + nbox * kBoxBytes));
-            tma_load_2d(a_s, &tm_h, full, kb * kKB, nt * kM, pol_h);
-            for (int j = 0; j < nbox; ++j)
-              tma_load_2d(b_s + j * kBoxBytes, &tm_w, full, kb * kKB, v0 + j * kLmBoxRows, pol_w);
+            const uint32_t a_s = base + stage * slot;
+            const uint32_t b_s = a_s + lm_a_bytes(p.a_rows);
+            const int nk = min(kKbPerStage, nkb - kp * kKbPerStage);
+            mbar_expect_tx(full, static_cast<uint32_t>(nk * (a_blk + ng * kGroupBytes)));
+            for (int kk = 0; kk < nk; ++kk) {
+              const int kx = (kp * kKbPerStage + kk) * kKB;
+              tma_load_2d(a_s + kk * a_blk, &tm_h, full, kx, nt * kM, pol_h);
+              int j = 0;
+              for (; j + 1 < ng; j += 2)
+                tma_load_2d(b_s + kk * kBTile + j * kGroupBytes, &tm_w64, full, kx,
+                            v0 + j * kLmBoxRows, pol_w);
+              if (j < ng)
+                tma_load_2d(b_s + kk * kBTile + j * kGroupBytes, &tm_w32, full, kx,
+                            v0 + j * kLmBoxRows, pol_w);
+            }
           }
           __syncwarp();
           if (++stage == kLmStages) {
@@ -214,7 +242,7 @@ __global__ void __launch_bounds__(192, 1)
         }
         tc_fence_after();
         const uint32_t d = tmem + static_cast<uint32_t>(acc * kLmTileN);
-        for (int kb = 0; kb < nkb; ++kb) {
+        for (int kp = 0; kp < nkp; ++kp) {
           ok = __shfl_sync(0xffffffffu, mbar_wait(smem_u32(&s_full[stage]), ph), 0);
           if (!ok || s_abort) {
             ok = false;
@@ -222,12 +250,16 @@ __global__ void __launch_bounds__(192, 1)
           }
           tc_fence_after();
           if (lane == 0) {
-            const uint32_t a_s = base + stage * kStage;
-            const uint32_t b_s = a_s + kATile;
+            const uint32_t a_s = base + stage * slot;
+            const uint32_t b_s = a_s + lm_a_bytes(p.a_rows);
+            const int nk = min(kKbPerStage, nkb - kp * kKbPerStage);
+            for (int kk = 0; kk < nk; ++kk) {
 #pragma unroll
-            for (int k = 0; k < kKB / 16; ++k)
-              tc_mma(d, sw128_desc(a_s + 32 * k), sw128_desc(b_s + 32 * k), idesc,
-                     (kb | k) != 0 ? 1u : 0u);
+              for (int k = 0; k < kKB / 16; ++k)
+                tc_mma(d, sw128_desc(a_s + kk * a_blk + 32 * k),
+                       sw128_desc(b_s + kk * kBTile + 32 * k), idesc,
+                       (kp | kk | k) != 0 ? 1u : 0u);
+            }
             tc_commit(smem_u32(&s_empty[stage]));
           }
           __syncwarp();
@@ -308,14 +340,19 @@ __global__ void __launch_bounds__(192, 1)
 
 }  // namespace
 
-size_t lmhead_tc_smem_bytes() { return 1024 + static_cast<size_t>(kLmStages) * kStage; }
+size_t lmhead_tc_smem_bytes(int a_rows) {
+  return 1024 + static_cast<size_t>(kLmStages) * lm_slot_bytes(a_rows);
+}
 
 cudaError_t launch_lmhead_bf16(const LmParams& p, const CUtensorMap& tm_hidden,
-                               const CUtensorMap& tm_w, cudaStream_t s) {
-  const size_t smem = lmhead_tc_smem_bytes();
+                               const CUtensorMap& tm_w64, const CUtensorMap& tm_w32,
+                               cudaStream_t s) {
+  if (p.a_rows < 8 || p.a_rows > kM || p.a_rows % 8) return cudaErrorInvalidValue;
+  const size_t smem = lmhead_tc_smem_bytes(p.a_rows);
   cudaError_t err = set_smem_attrs(lmhead_tc_kernel, smem);
   if (err != cudaSuccess) return err;
-  return launch_pdl(lmhead_tc_kernel, dim3(p.g_lm), dim3(192), smem, s, tm_hidden, tm_w, p);
+  return launch_pdl(lmhead_tc_kernel, dim3(p.g_lm), dim3(192), smem, s, tm_hidden, tm_w64,
+                    tm_w32, p);
 }
 
 }  // namespace asd
