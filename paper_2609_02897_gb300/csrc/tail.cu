@@ -49,7 +49,9 @@ __global__ void __launch_bounds__(kTailThreads) tail_kernel(const TailParams p) 
   __shared__ int s_path[kMaxNodes];
   __shared__ int s_maxd, s_len, s_skip;
 
-  pdl_wait();  // every earlier kernel of the step has completed
+  // Until pdl_wait() this kernel reads only caller inputs (cu_nodes, parent,
+  // tokens): no kernel of the call writes them, and every call starts behind
+  // a stream-ordered memset, so they are final even before the wait.
   const int b = blockIdx.x;
   const int i = threadIdx.x;
   const int warp = i >> 5, lane = i & 31;
@@ -57,6 +59,7 @@ __global__ void __launch_bounds__(kTailThreads) tail_kernel(const TailParams p) 
   const int e = p.cu_nodes[b + 1];
   const bool seq_ok = (s >= 0) && (e > s) && (e <= p.T) && (e - s <= p.max_nodes);
   if (!seq_ok) {
+    pdl_wait();
     if (i == 0) {
       set_status(p.status, ASD_ERR_TREE);
       if (p.mode & kTailWalk) {
@@ -78,13 +81,32 @@ __global__ void __launch_bounds__(kTailThreads) tail_kernel(const TailParams p) 
     s_par[i] = okn ? par : -1;
     s_tok[i] = p.tokens ? p.tokens[s + i] : 0;
   }
+  if (i == 0) {
+    s_maxd = 0;
+    s_len = 0;
+  }
   const int tree_bad = __syncthreads_or(!okn);
+  // node depths for the walk need the tree alone
+  if ((p.mode & kTailWalk) && !tree_bad && i < n) {
+    int d = 0, u = i;
+    while (s_par[u] >= 0) {
+      u = s_par[u];
+      ++d;
+    }
+    s_dep[i] = d;
+    s_h[i] = 1;
+    s_bc[i] = INT_MAX;
+    atomicMax(&s_maxd, d);
+  }
+
+  pdl_wait();  // every earlier kernel of the call has completed
   const int flags = p.seq_flags ? p.seq_flags[b] : 0;
+  // the drafted token's logit, loaded alongside the partials below
+  const float l_draft_i =
+      ((p.mode & kTailFinalize) && !tree_bad && i > 0 && i < n) ? p.l_draft[s + i] : 0.f;
   if (i == 0) {
     if (tree_bad) set_status(p.status, ASD_ERR_TREE);
     s_skip = (tree_bad || flags) ? 1 : 0;
-    s_maxd = 0;
-    s_len = 0;
   }
 
   // ---------------------------------------------------------------- finalize
@@ -126,7 +148,7 @@ __global__ void __launch_bounds__(kTailThreads) tail_kernel(const TailParams p) 
       float ratio = __int_as_float(0x7fc00000);
       if (i > 0) {
         const int pp = s_par[i];
-        const float d = p.l_draft[s + i] - s_max[pp];
+        const float d = l_draft_i - s_max[pp];
         const bool strict = s_tok[i] == s_arg[pp];
         ratio = expf(d);
         acc = (strict || d >= p.ln_tau) ? 1 : 0;
@@ -146,18 +168,6 @@ __global__ void __launch_bounds__(kTailThreads) tail_kernel(const TailParams p) 
   // -------------------------------------------------------------------- walk
   if (p.mode & kTailWalk) {
     if (!s_skip) {
-      if (i < n) {
-        int d = 0, u = i;
-        while (s_par[u] >= 0) {
-          u = s_par[u];
-          ++d;
-        }
-        s_dep[i] = d;
-        s_h[i] = 1;
-        s_bc[i] = INT_MAX;
-        atomicMax(&s_maxd, d);
-      }
-      __syncthreads();
       for (int dd = s_maxd; dd >= 1; --dd) {
         if (i < n && s_dep[i] == dd && s_acc[i]) atomicMax(&s_h[s_par[i]], s_h[i] + 1);
         __syncthreads();
