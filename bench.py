@@ -38,7 +38,7 @@ STAGES = ("prep", "lmhead", "attention", "tail")   # order of the stage events
 # DRAM bytes (read + write) of one LM-head launch on this workload, from the
 # ncu capture summarised in profiles/verify_step_llama8b_b1_ctx2048_tree60.md;
 # set to None whenever lmhead_tc.cu changes until it is captured again.
-LMHEAD_TRAFFIC_BYTES = 1054413264
+LMHEAD_TRAFFIC_BYTES = None
 
 
 def parse():
@@ -50,6 +50,8 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
+    ap.add_argument("--lm-layout", default="packed", choices=["packed", "rows"],
+                    help="LM-head weight as packed once at load (default) or as [V, K] rows")
     return ap.parse_args()
 
 
@@ -280,10 +282,19 @@ def run_asd(args):
     inputs = dict(q=f(wl.q), tree_k=f(wl.tree_k), tree_v=f(wl.tree_v), hidden=f(wl.hidden),
                   tokens=i(wl.tokens), parent=i(wl.parent), cu_nodes=i(wl.cu_nodes),
                   ctx_len=i(wl.ctx_len))
-    w_lm = f(wl.w)
     k_cache, v_cache = f(wl.k_cache), f(wl.v_cache)
+    packed = args.lm_layout == "packed"
     dims = asd.make_dims(wl.B, wl.Hq, wl.Hkv, wl.D, wl.hidden_dim, wl.vocab, asd.ASD_BF16, 0,
-                         wl.ctx_max, 0, wl.T, wl.max_path)
+                         wl.ctx_max, 0, wl.T, wl.max_path,
+                         asd.ASD_LM_PACKED if packed else asd.ASD_LM_ROWS)
+    w_lm = f(wl.w)
+    if packed:
+        # model load: the LM-head weight is repacked once into the streaming layout
+        w_rows = w_lm
+        w_lm = asd.pack_lm_head(dims, w_rows)
+        torch.cuda.synchronize()
+        del w_rows
+        torch.cuda.empty_cache()
     step = asd.VerifyStep(dims, wl.T, device=device)
     step.bind(w_lm=w_lm, k_cache=k_cache, v_cache=v_cache, tau=TAU, **inputs)
     stream = torch.cuda.current_stream()
@@ -383,6 +394,8 @@ def run_asd(args):
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic (seeded; Llama-3.1-8B-shaped tensors, random weights)",
         "config": workload_config(wl),
+        "lm_head_weight": ("packed once at load by asd_pack_lm_head (same bytes, streaming order)"
+                           if packed else "[vocab, hidden] rows"),
         "hbm_gbs": sb / (ms * 1e-3) / 1e9, "hbm_frac_of_" + peak_kind: sb / (ms * 1e-3) / 1e9 / peak,
         "roofline": {"kernel": "lmhead_tc_kernel", "bound": "hbm", "achieved": achieved,
                      "peak": peak, "unit": "GB/s", "frac": achieved / peak,

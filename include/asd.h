@@ -53,7 +53,7 @@
 extern "C" {
 #endif
 
-#define ASD_ABI_VERSION 1
+#define ASD_ABI_VERSION 2
 #define ASD_MAX_TREE_NODES 128
 #define ASD_NUM_STAGE_EVENTS 5
 
@@ -72,6 +72,12 @@ typedef enum asd_status {
 
 typedef enum asd_dtype { ASD_F32 = 0, ASD_BF16 = 1 } asd_dtype;
 
+/* Layout of the LM-head weight passed as w_lm. */
+typedef enum asd_lm_layout {
+  ASD_LM_ROWS = 0,   /* [vocab, hidden] row-major (HF lm_head.weight)            */
+  ASD_LM_PACKED = 1  /* bf16 only: the buffer written by asd_pack_lm_head        */
+} asd_lm_layout;
+
 /* Shapes of one verify step.  All fields are int32. */
 typedef struct asd_dims {
   int32_t batch;        /* B: number of sequences (trees)                      */
@@ -89,6 +95,7 @@ typedef struct asd_dims {
   int32_t max_nodes;    /* upper bound on nodes per tree, 1..128               */
   int32_t max_path;     /* columns of the path output, >= longest root-to-leaf
                            path (nodes, root included)                         */
+  int32_t lm_head_layout; /* asd_lm_layout of w_lm                             */
 } asd_dims;
 
 /* Bytes of device workspace that the calls below need for `total_nodes`
@@ -131,7 +138,8 @@ asd_status asd_tree_attention(const asd_dims* dims, const void* q, const void* k
  *             ratio[c] = exp(l_draft[c] - row_max[p])  (Eq. 1),
  *             accept[c] = tokens[c] == row_argmax[p]  ||  ratio >= tau.
  * Roots: accept = 1, l_draft = ratio = NaN.  Outputs are [T] arrays
- * (float32 / int32 / uint8).
+ * (float32 / int32 / uint8).  With dims->lm_head_layout = ASD_LM_PACKED,
+ * w_lm is a buffer from asd_pack_lm_head (same results, bit for bit).
  */
 asd_status asd_lmhead_margin(const asd_dims* dims, const void* hidden, const void* w_lm,
                              const int32_t* tokens, const int32_t* parent,
@@ -139,6 +147,27 @@ asd_status asd_lmhead_margin(const asd_dims* dims, const void* hidden, const voi
                              float* row_max, int32_t* row_argmax, float* row_lse,
                              float* l_draft, float* ratio, uint8_t* accept, void* workspace,
                              size_t workspace_bytes, void* stream);
+
+/*
+ * Streaming layout of the LM-head weight (no counterpart in the paper: a
+ * one-time repacking at model load that lets the LM head read W as one
+ * contiguous stream per SM instead of 128-byte pieces of 128 rows at a time,
+ * which HBM serves measurably slower).
+ * asd_lm_head_packed_bytes: size of the packed buffer for dims (bf16 only;
+ *   0 if the dims are invalid or fp32): 256 header bytes + W rounded up to
+ *   32 rows and 64 columns.
+ * asd_pack_lm_head: reads w [vocab, hidden] bf16 row-major and writes
+ *   w_packed (device, 256-byte aligned, packed_bytes >= the size above) on
+ *   `stream`.  The order depends on the SM count of the current device: use
+ *   the buffer on a device of the same kind, with the same vocab and hidden;
+ *   otherwise the LM head records ASD_ERR_SHAPE in the status word (its
+ *   outputs are then unspecified).  w and w_packed must not overlap.
+ *   Host errors: ASD_ERR_INVALID_ARG (null / misaligned pointers),
+ *   ASD_ERR_SHAPE (dims, fp32), ASD_ERR_WORKSPACE (packed_bytes too small).
+ */
+size_t asd_lm_head_packed_bytes(const asd_dims* dims);
+asd_status asd_pack_lm_head(const asd_dims* dims, const void* w, void* w_packed,
+                            size_t packed_bytes, void* stream);
 
 /*
  * Accepted path (step 3; Sec. 3.2 and Fig. 1: verification commits the

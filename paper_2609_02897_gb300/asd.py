@@ -20,6 +20,7 @@ if not os.path.exists(_LIB_PATH):
 _lib = ctypes.CDLL(_LIB_PATH)
 
 ASD_F32, ASD_BF16 = 0, 1
+ASD_LM_ROWS, ASD_LM_PACKED = 0, 1
 MAX_TREE_NODES = 128
 NUM_STAGE_EVENTS = 5
 STATUS = {0: "ASD_OK", 1: "ASD_ERR_INVALID_ARG", 2: "ASD_ERR_SHAPE", 3: "ASD_ERR_TREE",
@@ -27,7 +28,8 @@ STATUS = {0: "ASD_OK", 1: "ASD_ERR_INVALID_ARG", 2: "ASD_ERR_SHAPE", 3: "ASD_ERR
           7: "ASD_ERR_CUDA", 8: "ASD_ERR_TIMEOUT", 9: "ASD_ERR_UNSUPPORTED"}
 EXPORTS = ["asd_workspace_bytes", "asd_tree_attention", "asd_lmhead_margin", "asd_accept_path",
            "asd_kv_compact", "asd_verify_step", "asd_get_device_status", "asd_status_string",
-           "asd_abi_version", "asd_lmhead_margin_noalloc"]
+           "asd_abi_version", "asd_lmhead_margin_noalloc", "asd_lm_head_packed_bytes",
+           "asd_pack_lm_head"]
 
 
 class AsdError(RuntimeError):
@@ -40,7 +42,7 @@ class AsdError(RuntimeError):
 class Dims(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int32) for n in (
         "batch", "num_q_heads", "num_kv_heads", "head_dim", "hidden", "vocab", "dtype",
-        "page_size", "ctx_max", "num_pages", "max_nodes", "max_path")]
+        "page_size", "ctx_max", "num_pages", "max_nodes", "max_path", "lm_head_layout")]
 
 
 _vp = ctypes.c_void_p
@@ -84,6 +86,10 @@ _lib.asd_lmhead_margin_noalloc.argtypes = [_P] + [_vp] * 5 + [ctypes.c_int32, ct
     _vp] * 6 + [_vp, _vp]
 _lib.asd_get_device_status.restype = ctypes.c_int
 _lib.asd_get_device_status.argtypes = [_vp, ctypes.POINTER(ctypes.c_int32), _vp]
+_lib.asd_lm_head_packed_bytes.restype = ctypes.c_size_t
+_lib.asd_lm_head_packed_bytes.argtypes = [_P]
+_lib.asd_pack_lm_head.restype = ctypes.c_int
+_lib.asd_pack_lm_head.argtypes = [_P, _vp, _vp, ctypes.c_size_t, _vp]
 
 
 def lib_path() -> str:
@@ -95,9 +101,9 @@ def abi_version() -> int:
 
 
 def make_dims(batch, num_q_heads, num_kv_heads, head_dim, hidden, vocab, dtype, page_size,
-              ctx_max, num_pages, max_nodes, max_path) -> Dims:
+              ctx_max, num_pages, max_nodes, max_path, lm_head_layout=0) -> Dims:
     return Dims(batch, num_q_heads, num_kv_heads, head_dim, hidden, vocab, dtype, page_size,
-                ctx_max, num_pages, max_nodes, max_path)
+                ctx_max, num_pages, max_nodes, max_path, lm_head_layout)
 
 
 def _ptr(t: Optional[torch.Tensor]):
@@ -126,6 +132,26 @@ def asd_workspace_bytes(dims: Dims, total_nodes: int) -> int:
     if n == 0:
         raise AsdError(2, "asd_workspace_bytes")
     return n
+
+
+def asd_lm_head_packed_bytes(dims: Dims) -> int:
+    n = int(_lib.asd_lm_head_packed_bytes(ctypes.byref(dims)))
+    if n == 0:
+        raise AsdError(2, "asd_lm_head_packed_bytes")
+    return n
+
+
+def asd_pack_lm_head(dims: Dims, w: torch.Tensor, w_packed: torch.Tensor, stream=None):
+    _check(_lib.asd_pack_lm_head(ctypes.byref(dims), _ptr(w), _ptr(w_packed), w_packed.numel(),
+                                 _stream(stream)), "asd_pack_lm_head")
+
+
+def pack_lm_head(dims: Dims, w: torch.Tensor, stream=None) -> torch.Tensor:
+    """A new device buffer holding w in the LM head's packed streaming layout
+    (use it with dims.lm_head_layout = ASD_LM_PACKED)."""
+    out = torch.empty(asd_lm_head_packed_bytes(dims), dtype=torch.uint8, device=w.device)
+    asd_pack_lm_head(dims, w, out, stream)
+    return out
 
 
 def alloc_workspace(dims: Dims, total_nodes: int, device="cuda") -> torch.Tensor:

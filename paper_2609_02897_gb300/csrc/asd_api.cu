@@ -45,6 +45,14 @@ bool make_tmap_bf16(CUtensorMap* tm, const void* base, uint64_t cols, uint64_t r
              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+}  // namespace
+
+int asd::lm_ranges(int vocab, int nsm) {
+  return std::max(1, std::min(std::min(nsm, kMaxLmRanges), (vocab + kLmBoxRows - 1) / kLmBoxRows));
+}
+
+namespace {
+
 int device_sm_count() {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return 0;
@@ -78,6 +86,8 @@ bool dims_ok(const asd_dims* d) {
   }
   if (d->max_nodes < 1 || d->max_nodes > ASD_MAX_TREE_NODES) return false;
   if (d->max_path < 1) return false;
+  if (d->lm_head_layout != ASD_LM_ROWS && d->lm_head_layout != ASD_LM_PACKED) return false;
+  if (d->lm_head_layout == ASD_LM_PACKED && d->dtype != ASD_BF16) return false;
   return true;
 }
 
@@ -89,7 +99,7 @@ bool nodes_ok(const asd_dims* d, int32_t total_nodes) {
 WsLayout layout(const asd_dims& d, int T, int nsm) {
   WsLayout L{};
   const int G = d.num_q_heads / d.num_kv_heads;
-  L.g_lm = std::max(1, std::min(std::min(nsm, kMaxLmRanges), (d.vocab + kLmBoxRows - 1) / kLmBoxRows));
+  L.g_lm = lm_ranges(d.vocab, nsm);
   // context splits: at most one attention CTA per SM (in a verify step each
   // shares its SM with an LM-head CTA), at most kMaxAttnParts (the splits of a
   // row block form one thread-block cluster); the last non-empty split of a
@@ -246,12 +256,16 @@ asd_status run_lmhead(const Ctx& c, const void* hidden, const void* w, float* l_
   p.a_rows = std::min(128, (c.T + 7) / 8 * 8);
   cudaError_t err;
   if (d.dtype == ASD_BF16) {
-    CUtensorMap th, tw64, tw32;
-    if (!make_tmap_bf16(&th, hidden, d.hidden, c.T, static_cast<uint32_t>(p.a_rows)) ||
-        !make_tmap_bf16(&tw64, w, d.hidden, d.vocab, 2 * kLmBoxRows) ||
-        !make_tmap_bf16(&tw32, w, d.hidden, d.vocab, kLmBoxRows))
+    LmMaps m{};
+    if (!make_tmap_bf16(&m.h, hidden, d.hidden, c.T, static_cast<uint32_t>(p.a_rows)))
       return ASD_ERR_CUDA;
-    err = launch_lmhead_bf16(p, th, tw64, tw32, c.st);
+    if (d.lm_head_layout == ASD_LM_PACKED) {
+      p.w_packed = static_cast<const uint8_t*>(w);
+    } else if (!make_tmap_bf16(&m.w64, w, d.hidden, d.vocab, 2 * kLmBoxRows) ||
+               !make_tmap_bf16(&m.w32, w, d.hidden, d.vocab, kLmBoxRows)) {
+      return ASD_ERR_CUDA;
+    }
+    err = launch_lmhead_bf16(p, m, c.st);
   } else {
     err = launch_lmhead_f32(p, c.st);
   }
@@ -306,6 +320,29 @@ const char* asd_status_string(int32_t s) {
     case ASD_ERR_UNSUPPORTED: return "unsupported device or feature";
     default: return "unknown status";
   }
+}
+
+size_t asd_lm_head_packed_bytes(const asd_dims* dims) {
+  if (!dims_ok(dims) || dims->dtype != ASD_BF16) return 0;
+  return lm_packed_bytes(dims->vocab, dims->hidden);
+}
+
+asd_status asd_pack_lm_head(const asd_dims* dims, const void* w, void* w_packed,
+                            size_t packed_bytes, void* stream) {
+  if (!dims || !w || !w_packed) return ASD_ERR_INVALID_ARG;
+  if (!dims_ok(dims) || dims->dtype != ASD_BF16) return ASD_ERR_SHAPE;
+  if (!aligned16(w) || (reinterpret_cast<uintptr_t>(w_packed) & 255u)) return ASD_ERR_INVALID_ARG;
+  const size_t need = lm_packed_bytes(dims->vocab, dims->hidden);
+  if (packed_bytes < need) return ASD_ERR_WORKSPACE;
+  const uintptr_t a0 = reinterpret_cast<uintptr_t>(w), a1 = a0 + 2ull * dims->vocab * dims->hidden;
+  const uintptr_t b0 = reinterpret_cast<uintptr_t>(w_packed), b1 = b0 + need;
+  if (a0 < b1 && b0 < a1) return ASD_ERR_INVALID_ARG;
+  const int nsm = device_sm_count();
+  if (nsm <= 0) return ASD_ERR_CUDA;
+  return launch_lm_pack(w, w_packed, dims->vocab, dims->hidden, lm_ranges(dims->vocab, nsm),
+                        static_cast<cudaStream_t>(stream)) == cudaSuccess
+             ? ASD_OK
+             : ASD_ERR_CUDA;
 }
 
 size_t asd_workspace_bytes(const asd_dims* dims, int32_t total_nodes) {
@@ -532,7 +569,7 @@ void* noalloc_scratch() {
 // Regions of the LM-head path only (no attention partials).
 WsLayout lmhead_only_layout(const asd_dims& d, int T, int nsm) {
   WsLayout L{};
-  L.g_lm = std::max(1, std::min(std::min(nsm, kMaxLmRanges), (d.vocab + kLmBoxRows - 1) / kLmBoxRows));
+  L.g_lm = lm_ranges(d.vocab, nsm);
   size_t off = 0;
   L.status = off;      off = align256(off + 16);
   L.seq_flags = off;   off = align256(off + 4 * static_cast<size_t>(d.batch));

@@ -100,16 +100,46 @@ struct LmParams {
   int T, K, V, g_lm;
   int a_rows;               // node rows per hidden-state TMA box: min(128, T rounded to 8);
                             // accumulator rows past it belong to no node
+  const uint8_t* w_packed;  // W in the packed streaming layout, or null ([V, K] rows via TMA)
 };
 constexpr int kLmStages = 3;       // 3 x 48 KB (a_rows <= 64): room for an attention CTA
 constexpr int kLmTileN = 128;      // vocabulary rows per MMA tile
 constexpr int kLmBoxRows = 32;     // vocabulary rows per range group (and per small TMA box)
 size_t lmhead_tc_smem_bytes(int a_rows);
+// Tensor maps of the bf16 LM head (128-byte swizzle, 64-element inner boxes):
+// h: hidden [T, K], box a_rows rows; w64 / w32: W [V, K], boxes of 64 and 32
+// rows (unused with a packed weight).
+struct LmMaps {
+  CUtensorMap h, w64, w32;
+};
 // bf16 path: tcgen05/TMEM GEMM with the fused max/argmax/sum-exp/l_draft epilogue.
-// tm_w64 / tm_w32: tensor maps over W [V, K] with boxes of 64 and 32 rows.
-cudaError_t launch_lmhead_bf16(const LmParams& p, const CUtensorMap& tm_hidden,
-                               const CUtensorMap& tm_w64, const CUtensorMap& tm_w32,
-                               cudaStream_t s);
+cudaError_t launch_lmhead_bf16(const LmParams& p, const LmMaps& maps, cudaStream_t s);
+
+// Vocabulary ranges of the LM head: range c of g covers the 32-row groups
+// [c * ngroups / g, (c + 1) * ngroups / g); each range is cut into tiles of
+// up to kLmTileN rows starting at its first group.
+__host__ __device__ inline int lm_range_begin(int c, int g, int ngroups) {
+  return static_cast<int>(static_cast<long long>(c) * ngroups / g);
+}
+int lm_ranges(int vocab, int nsm);
+
+// Packed streaming layout of the LM-head weight (asd_pack_lm_head): a header
+// of kLmPackHeader bytes, then for every tile in range order and every
+// k-block kb, the tile's rows (ng whole 32-row groups, zeros past V and past
+// K) x 128 bytes with the 128-byte swizzle applied (16-byte chunk c of row r
+// at chunk c ^ (r & 7)).  The block of a tile starting at group g0 for
+// k-block kb begins at byte kLmPackHeader + 4096 * (nkb * g0 + kb * ng), so a
+// stage's two k-blocks are one contiguous run.
+constexpr uint32_t kLmPackMagic = 0x57445341u;  // "ASDW"
+constexpr uint32_t kLmPackVersion = 1;
+constexpr int kLmPackHeader = 256;
+struct LmPackHeader {
+  uint32_t magic, version;
+  int32_t vocab, hidden, ranges;
+};
+size_t lm_packed_bytes(int vocab, int hidden);
+cudaError_t launch_lm_pack(const void* w, void* w_packed, int vocab, int hidden, int ranges,
+                           cudaStream_t s);
 cudaError_t launch_lmhead_f32(const LmParams& p, cudaStream_t s);
 
 // --------------------------------------- finalize / accepted path / K/V commit

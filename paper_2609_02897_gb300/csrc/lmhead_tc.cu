@@ -117,9 +117,7 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
 }
 
 __global__ void __launch_bounds__(192, 1)
-    lmhead_tc_kernel(const __grid_constant__ CUtensorMap tm_h,
-                     const __grid_constant__ CUtensorMap tm_w64,
-                     const __grid_constant__ CUtensorMap tm_w32, const LmParams p) {
+    lmhead_tc_kernel(const __grid_constant__ LmMaps maps, const LmParams p) {
   extern __shared__ uint8_t smem_raw[];
   __shared__ __align__(8) uint64_t s_full[kLmStages];
   __shared__ __align__(8) uint64_t s_empty[kLmStages];
@@ -127,6 +125,7 @@ __global__ void __launch_bounds__(192, 1)
   __shared__ __align__(8) uint64_t s_tempty[2];
   __shared__ uint32_t s_tmem;
   __shared__ volatile int s_abort;
+  __shared__ int s_pack_bad;
 
   // W and the hidden states are inputs of the step, not results of earlier
   // kernels: only the epilogue (children lists, l_draft) waits for them
@@ -135,11 +134,10 @@ __global__ void __launch_bounds__(192, 1)
 
   // this CTA's vocabulary range, in whole groups of kLmBoxRows rows
   const int ngroups = (p.V + kLmBoxRows - 1) / kLmBoxRows;
-  const int gs = static_cast<int>(static_cast<long long>(blockIdx.x) * ngroups / p.g_lm);
-  const int ge = static_cast<int>(static_cast<long long>(blockIdx.x + 1) * ngroups / p.g_lm);
+  const int gs = lm_range_begin(blockIdx.x, p.g_lm, ngroups);
+  const int ge = lm_range_begin(blockIdx.x + 1, p.g_lm, ngroups);
   const int vs = gs * kLmBoxRows;
   const int ve = min(p.V, ge * kLmBoxRows);
-  const int nvt = ve > vs ? (ve - vs + kLmTileN - 1) / kLmTileN : 0;
   const int nnt = (p.T + kM - 1) / kM;
   const int nkb = (p.K + kKB - 1) / kKB;
   const int nkp = (nkb + kKbPerStage - 1) / kKbPerStage;   // stages per tile
@@ -159,6 +157,16 @@ __global__ void __launch_bounds__(192, 1)
       mbar_init(smem_u32(&s_tempty[a]), 4);
     }
     s_abort = 0;
+    // a packed weight must come from asd_pack_lm_head for this vocabulary,
+    // width and range count; otherwise nothing is loaded and the error recorded
+    int bad = 0;
+    if (p.w_packed) {
+      const LmPackHeader* h = reinterpret_cast<const LmPackHeader*>(p.w_packed);
+      bad = (h->magic != kLmPackMagic || h->version != kLmPackVersion || h->vocab != p.V ||
+             h->hidden != p.K || h->ranges != p.g_lm);
+      if (bad) set_status(p.status, ASD_ERR_SHAPE);
+    }
+    s_pack_bad = bad;
     fence_mbar_init();
   }
   if (warp == 1) {
@@ -169,14 +177,18 @@ __global__ void __launch_bounds__(192, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = s_tmem;
+  // vocabulary tiles of this CTA (none when a packed weight does not match)
+  const int nvt = (ve > vs && !s_pack_bad) ? (ve - vs + kLmTileN - 1) / kLmTileN : 0;
 
   if (warp == 0) {
     // ------------------------------------------------------------ TMA producer
     uint64_t pol_w = 0, pol_h = 0;
     if (lane == 0) {
-      prefetch_tmap(&tm_h);
-      prefetch_tmap(&tm_w64);
-      prefetch_tmap(&tm_w32);
+      prefetch_tmap(&maps.h);
+      if (!p.w_packed) {
+        prefetch_tmap(&maps.w64);
+        prefetch_tmap(&maps.w32);
+      }
       pol_w = l2_policy_evict_first();
       pol_h = l2_policy_evict_last();
     }
@@ -199,16 +211,28 @@ __global__ void __launch_bounds__(192, 1)
             const uint32_t b_s = a_s + lm_a_bytes(p.a_rows);
             const int nk = min(kKbPerStage, nkb - kp * kKbPerStage);
             mbar_expect_tx(full, static_cast<uint32_t>(nk * (a_blk + ng * kGroupBytes)));
-            for (int kk = 0; kk < nk; ++kk) {
-              const int kx = (kp * kKbPerStage + kk) * kKB;
-              tma_load_2d(a_s + kk * a_blk, &tm_h, full, kx, nt * kM, pol_h);
-              int j = 0;
-              for (; j + 1 < ng; j += 2)
-                tma_load_2d(b_s + kk * kBTile + j * kGroupBytes, &tm_w64, full, kx,
-                            v0 + j * kLmBoxRows, pol_w);
-              if (j < ng)
-                tma_load_2d(b_s + kk * kBTile + j * kGroupBytes, &tm_w32, full, kx,
-                            v0 + j * kLmBoxRows, pol_w);
+            for (int kk = 0; kk < nk; ++kk)
+              tma_load_2d(a_s + kk * a_blk, &maps.h, full, (kp * kKbPerStage + kk) * kKB,
+                          nt * kM, pol_h);
+            if (p.w_packed) {
+              // both k-blocks of the stage are one contiguous run of the packed weight
+              const size_t off = kLmPackHeader +
+                                 static_cast<size_t>(kGroupBytes) *
+                                     (static_cast<size_t>(nkb) * (v0 / kLmBoxRows) +
+                                      static_cast<size_t>(kp * kKbPerStage) * ng);
+              bulk_load(b_s, p.w_packed + off, static_cast<uint32_t>(nk * ng * kGroupBytes), full,
+                        pol_w);
+            } else {
+              for (int kk = 0; kk < nk; ++kk) {
+                const int kx = (kp * kKbPerStage + kk) * kKB;
+                int j = 0;
+                for (; j + 1 < ng; j += 2)
+                  tma_load_2d(b_s + kk * kBTile + j * kGroupBytes, &maps.w64, full, kx,
+                              v0 + j * kLmBoxRows, pol_w);
+                if (j < ng)
+                  tma_load_2d(b_s + kk * kBTile + j * kGroupBytes, &maps.w32, full, kx,
+                              v0 + j * kLmBoxRows, pol_w);
+              }
             }
           }
           __syncwarp();
@@ -235,6 +259,10 @@ __global__ void __launch_bounds__(192, 1)
         const int v0 = vs + vt * kLmTileN;
         const int nrows = min(kLmTileN, ve - v0);
         const uint32_t idesc = idesc_bf16(kM, (nrows + 15) & ~15);
+        // the second k-block's W rows: a fixed slot, or right behind the first
+        // block's ng groups in the packed layout
+        const int b_kstride =
+            p.w_packed ? ((nrows + kLmBoxRows - 1) / kLmBoxRows) * kGroupBytes : kBTile;
         ok = __shfl_sync(0xffffffffu, mbar_wait(smem_u32(&s_tempty[acc]), aph ^ 1u), 0);
         if (!ok || s_abort) {
           ok = false;
@@ -257,7 +285,7 @@ __global__ void __launch_bounds__(192, 1)
 #pragma unroll
               for (int k = 0; k < kKB / 16; ++k)
                 tc_mma(d, sw128_desc(a_s + kk * a_blk + 32 * k),
-                       sw128_desc(b_s + kk * kBTile + 32 * k), idesc,
+                       sw128_desc(b_s + kk * b_kstride + 32 * k), idesc,
                        (kp | kk | k) != 0 ? 1u : 0u);
             }
             tc_commit(smem_u32(&s_empty[stage]));
@@ -340,19 +368,71 @@ __global__ void __launch_bounds__(192, 1)
 
 }  // namespace
 
+// One CTA per (32-row group g, k-block kb): copies that 4 KB block of W into
+// its place in the packed layout, swizzled, zeros past V.  Block (0, 0) also
+// writes the header.
+__global__ void __launch_bounds__(256) lm_pack_kernel(const __nv_bfloat16* w, uint8_t* out,
+                                                      int V, int K, int ranges) {
+  const int g = blockIdx.x, kb = blockIdx.y;
+  const int ngroups = gridDim.x, nkb = gridDim.y;
+  // the range holding group g, and its tile
+  int c = static_cast<int>(static_cast<long long>(g) * ranges / ngroups);
+  while (c + 1 < ranges && lm_range_begin(c + 1, ranges, ngroups) <= g) ++c;
+  while (c > 0 && lm_range_begin(c, ranges, ngroups) > g) --c;
+  const int gs = lm_range_begin(c, ranges, ngroups), ge = lm_range_begin(c + 1, ranges, ngroups);
+  const int tile_groups = kLmTileN / kLmBoxRows;
+  const int g0 = gs + ((g - gs) / tile_groups) * tile_groups;
+  const int ng = min(tile_groups, ge - g0);
+  const size_t blk = kLmPackHeader + static_cast<size_t>(kGroupBytes) *
+                                         (static_cast<size_t>(nkb) * g0 + static_cast<size_t>(kb) * ng +
+                                          (g - g0));
+  const int r = threadIdx.x >> 3, ch = threadIdx.x & 7;
+  const int row = g * kLmBoxRows + r, col = kb * kKB + ch * 8;
+  uint4 v = make_uint4(0u, 0u, 0u, 0u);
+  if (row < V && col < K)  // K % 8 == 0: a chunk is all in or all out
+    v = *reinterpret_cast<const uint4*>(w + static_cast<size_t>(row) * K + col);
+  *reinterpret_cast<uint4*>(out + blk + r * 128 + ((ch ^ (r & 7)) << 4)) = v;
+  if (g == 0 && kb == 0 && threadIdx.x < kLmPackHeader / 4) {
+    uint32_t word = 0;
+    switch (threadIdx.x) {
+      case 0: word = kLmPackMagic; break;
+      case 1: word = kLmPackVersion; break;
+      case 2: word = static_cast<uint32_t>(V); break;
+      case 3: word = static_cast<uint32_t>(K); break;
+      case 4: word = static_cast<uint32_t>(ranges); break;
+      default: break;
+    }
+    reinterpret_cast<uint32_t*>(out)[threadIdx.x] = word;
+  }
+}
+
 size_t lmhead_tc_smem_bytes(int a_rows) {
   return 1024 + static_cast<size_t>(kLmStages) * lm_slot_bytes(a_rows);
 }
 
-cudaError_t launch_lmhead_bf16(const LmParams& p, const CUtensorMap& tm_hidden,
-                               const CUtensorMap& tm_w64, const CUtensorMap& tm_w32,
-                               cudaStream_t s) {
+size_t lm_packed_bytes(int vocab, int hidden) {
+  const size_t ngroups = (static_cast<size_t>(vocab) + kLmBoxRows - 1) / kLmBoxRows;
+  const size_t nkb = (static_cast<size_t>(hidden) + kKB - 1) / kKB;
+  return kLmPackHeader + ngroups * nkb * kGroupBytes;
+}
+
+cudaError_t launch_lm_pack(const void* w, void* w_packed, int vocab, int hidden, int ranges,
+                           cudaStream_t s) {
+  const unsigned ngroups = static_cast<unsigned>((vocab + kLmBoxRows - 1) / kLmBoxRows);
+  const unsigned nkb = static_cast<unsigned>((hidden + kKB - 1) / kKB);
+  if (nkb > 65535u) return cudaErrorInvalidValue;
+  lm_pack_kernel<<<dim3(ngroups, nkb), 256, 0, s>>>(static_cast<const __nv_bfloat16*>(w),
+                                                    static_cast<uint8_t*>(w_packed), vocab,
+                                                    hidden, ranges);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_lmhead_bf16(const LmParams& p, const LmMaps& maps, cudaStream_t s) {
   if (p.a_rows < 8 || p.a_rows > kM || p.a_rows % 8) return cudaErrorInvalidValue;
   const size_t smem = lmhead_tc_smem_bytes(p.a_rows);
   cudaError_t err = set_smem_attrs(lmhead_tc_kernel, smem);
   if (err != cudaSuccess) return err;
-  return launch_pdl(lmhead_tc_kernel, dim3(p.g_lm), dim3(192), smem, s, tm_hidden, tm_w64,
-                    tm_w32, p);
+  return launch_pdl(lmhead_tc_kernel, dim3(p.g_lm), dim3(192), smem, s, maps, p);
 }
 
 }  // namespace asd

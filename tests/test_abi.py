@@ -24,7 +24,7 @@ def _declared():
 
 def test_every_declared_function_is_exported(lib):
     names = _declared()
-    assert len(names) == 10, names
+    assert len(names) == 12, names
     for n in names:
         assert hasattr(lib, n), n
 
@@ -34,7 +34,7 @@ def test_binding_names_match_header():
     build.build()
     from paper_2609_02897_gb300 import asd
     assert sorted(asd.EXPORTS) == _declared()
-    assert asd.abi_version() == 1
+    assert asd.abi_version() == 2
 
 
 def test_host_checks_without_gpu(lib):
@@ -52,3 +52,26 @@ def test_host_checks_without_gpu(lib):
     assert lib.asd_lmhead_margin(*args, f(float("nan")), *outs) == 1
     lib.asd_status_string.restype = ctypes.c_char_p
     assert lib.asd_status_string(3) == b"malformed draft tree"
+
+
+def test_packed_lm_head_host_checks(lib):
+    """Size of the packed LM-head weight (256 header bytes + W rounded up to
+    32 rows and 64 columns) and the packing call's host-side rejections,
+    answered before any CUDA call."""
+    from paper_2609_02897_gb300 import asd
+    V, K = 1000, 200            # 32 groups (1024 rows), 4 k-blocks (256 columns)
+    d = asd.make_dims(1, 4, 4, 64, K, V, asd.ASD_BF16, 0, 64, 0, 8, 5)
+    assert asd.asd_lm_head_packed_bytes(d) == 256 + 32 * 4 * 4096
+    f = asd.make_dims(1, 4, 4, 64, K, V, asd.ASD_F32, 0, 64, 0, 8, 5)
+    assert lib.asd_lm_head_packed_bytes(ctypes.byref(f)) == 0
+    pk = asd.make_dims(1, 4, 4, 64, K, V, asd.ASD_F32, 0, 64, 0, 8, 5, asd.ASD_LM_PACKED)
+    assert lib.asd_workspace_bytes(ctypes.byref(pk), 8) == 0     # packed W is bf16 only
+    bad = asd.make_dims(1, 4, 4, 64, K, V, asd.ASD_BF16, 0, 64, 0, 8, 5, 7)
+    assert lib.asd_workspace_bytes(ctypes.byref(bad), 8) == 0    # unknown layout
+    fn = asd._lib.asd_pack_lm_head
+    w, out = ctypes.c_void_p(1 << 20), ctypes.c_void_p(1 << 30)
+    assert fn(ctypes.byref(d), None, out, 1 << 30, None) == 1
+    assert fn(ctypes.byref(f), w, out, 1 << 30, None) == 2
+    assert fn(ctypes.byref(d), w, ctypes.c_void_p((1 << 30) + 16), 1 << 30, None) == 1  # alignment
+    assert fn(ctypes.byref(d), w, out, 4096, None) == 6                                 # too small
+    assert fn(ctypes.byref(d), w, ctypes.c_void_p((1 << 20) + 256), 1 << 30, None) == 1  # overlap
