@@ -38,7 +38,7 @@ STAGES = ("prep", "lmhead", "attention", "tail")   # order of the stage events
 # DRAM bytes (read + write) of one LM-head launch on this workload, from the
 # ncu capture summarised in profiles/verify_step_llama8b_b1_ctx2048_tree60.md;
 # set to None whenever lmhead_tc.cu changes until it is captured again.
-LMHEAD_TRAFFIC_BYTES = None
+LMHEAD_TRAFFIC_BYTES = 1054301744
 
 
 def parse():
