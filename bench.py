@@ -50,6 +50,11 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
+    ap.add_argument("--config", type=int, default=CONFIG,
+                    help="workload number (synth.WORKLOADS); the default is the headline "
+                         "Llama-3.1-8B-shaped verify step, the others are for the record")
+    ap.add_argument("--tau", type=float, default=None,
+                    help="margin threshold (default: the workload's first)")
     ap.add_argument("--lm-layout", default="packed", choices=["packed", "rows"],
                     help="LM-head weight as packed once at load (default) or as [V, K] rows")
     return ap.parse_args()
@@ -64,30 +69,65 @@ def peaks():
         return 6800.0, "fallback"
 
 
+def tensor_peak():
+    """Dense bf16 TFLOP/s: the measured burst figure, else the fallback."""
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return float(json.load(f)["bf16_tflops"]), "measured"
+    except Exception:
+        return 1900.0, "fallback"
+
+
 def workload_config(wl):
+    if CONFIG == 2:
+        desc = ("llama3.1-8b-shaped verify step: batch 1, context 2048, 32 q / 8 kv heads, "
+                "head_dim 128, hidden 4096, vocab 128256, 60-node EAGLE-style tree "
+                "(depth<=8, top-k 10), tau 0.3, bf16")
+    else:
+        desc = (f"{wl.name}: batch {wl.B}, context {int(wl.ctx_len.min())}-{int(wl.ctx_len.max())}, "
+                f"{wl.Hq} q / {wl.Hkv} kv heads, head_dim {wl.D}, hidden {wl.hidden_dim}, "
+                f"vocab {wl.vocab}, {wl.T} tree nodes"
+                + (f", paged ({wl.page_size} tokens per page)" if wl.page_size else "")
+                + f", tau {TAU}, {wl.dtype}")
     return {
-        "workload": "llama3.1-8b-shaped verify step: batch 1, context 2048, 32 q / 8 kv heads, "
-                    "head_dim 128, hidden 4096, vocab 128256, 60-node EAGLE-style tree "
-                    "(depth<=8, top-k 10), tau 0.3, bf16",
+        "workload": desc,
         "batch": wl.B, "ctx": int(wl.ctx_len[0]), "tree_nodes": wl.T,
         "tree_depth": int(wl.max_path - 1), "tau": TAU,
         "l2": "inputs larger than L2: the 1.05 GB LM-head weight is streamed every step",
     }
 
 
+def esz(wl):
+    """Bytes per element of the workload's tensors."""
+    return 2 if wl.dtype == "bf16" else 4
+
+
 def lmhead_bytes(wl):
     """Algorithmic bytes of the LM-head kernel: W and the hidden states read once,
     per-row statistics written."""
-    return wl.vocab * wl.hidden_dim * 2 + wl.T * wl.hidden_dim * 2 + wl.T * 16
+    return (wl.vocab + wl.T) * wl.hidden_dim * esz(wl) + wl.T * 16
+
+
+def step_flops(wl):
+    """Algorithmic flops of one verify step: 4*Hq*D per (query node, visible key)
+    in attention, 2*hidden*V per LM-head row."""
+    import oracle
+    keys = 0
+    for b in range(wl.B):
+        s, e = int(wl.cu_nodes[b]), int(wl.cu_nodes[b + 1])
+        keys += (e - s) * int(wl.ctx_len[b])
+        keys += sum(len(oracle.ancestors_of(wl.parent[s:e], i)) for i in range(e - s))
+    return 4 * keys * wl.Hq * wl.D + 2 * wl.T * wl.hidden_dim * wl.vocab
 
 
 def step_bytes(wl, mean_path):
     """Algorithmic bytes of one verify step (every input read once, outputs written)."""
     ctx = int(wl.ctx_len.sum())
-    attn = (ctx * wl.Hkv * wl.D * 2 * 2            # context K and V
-            + wl.T * wl.Hkv * wl.D * 2 * 2        # tree K and V
-            + wl.T * wl.Hq * wl.D * 2 * 2)        # Q read, O written
-    commit = mean_path * wl.B * wl.Hkv * wl.D * 2 * 2 * 2
+    e = esz(wl)
+    attn = (ctx * wl.Hkv * wl.D * 2 * e            # context K and V
+            + wl.T * wl.Hkv * wl.D * 2 * e        # tree K and V
+            + wl.T * wl.Hq * wl.D * 2 * e)        # Q read, O written
+    commit = mean_path * wl.B * wl.Hkv * wl.D * 2 * 2 * e
     return attn + lmhead_bytes(wl) + commit
 
 
@@ -271,7 +311,8 @@ def run_asd(args):
     wl = synth.make_workload(CONFIG, rep=rank)
     synth.attach_tokens(wl, ranks_torch(wl, device))
     torch.cuda.empty_cache()
-    bf = torch.bfloat16
+    is_bf16 = wl.dtype == "bf16"
+    bf = torch.bfloat16 if is_bf16 else torch.float32
 
     def f(x):
         return torch.from_numpy(np.ascontiguousarray(x)).to(device=device, dtype=bf)
@@ -282,10 +323,13 @@ def run_asd(args):
     inputs = dict(q=f(wl.q), tree_k=f(wl.tree_k), tree_v=f(wl.tree_v), hidden=f(wl.hidden),
                   tokens=i(wl.tokens), parent=i(wl.parent), cu_nodes=i(wl.cu_nodes),
                   ctx_len=i(wl.ctx_len))
+    if wl.page_table is not None:
+        inputs["page_table"] = i(wl.page_table)
     k_cache, v_cache = f(wl.k_cache), f(wl.v_cache)
-    packed = args.lm_layout == "packed"
-    dims = asd.make_dims(wl.B, wl.Hq, wl.Hkv, wl.D, wl.hidden_dim, wl.vocab, asd.ASD_BF16, 0,
-                         wl.ctx_max, 0, wl.T, wl.max_path,
+    packed = args.lm_layout == "packed" and is_bf16   # the packed layout is bf16 only
+    dims = asd.make_dims(wl.B, wl.Hq, wl.Hkv, wl.D, wl.hidden_dim, wl.vocab,
+                         asd.ASD_BF16 if is_bf16 else asd.ASD_F32, wl.page_size,
+                         wl.ctx_max, wl.num_pages, int(np.diff(wl.cu_nodes).max()), wl.max_path,
                          asd.ASD_LM_PACKED if packed else asd.ASD_LM_ROWS)
     w_lm = f(wl.w)
     if packed:
@@ -295,7 +339,7 @@ def run_asd(args):
         torch.cuda.synchronize()
         del w_rows
         torch.cuda.empty_cache()
-    step = asd.VerifyStep(dims, wl.T, device=device)
+    step = asd.VerifyStep(dims, wl.T, device=device, attn_dtype=bf)
     step.bind(w_lm=w_lm, k_cache=k_cache, v_cache=v_cache, tau=TAU, **inputs)
     stream = torch.cuda.current_stream()
 
@@ -388,20 +432,41 @@ def run_asd(args):
     lmb = lmhead_bytes(wl)
     achieved = lmb / (lm_ms * 1e-3) / 1e9
     sb = step_bytes(wl, mean_path)
+    fl = step_flops(wl)
+    tpk, tpk_kind = tensor_peak()
+    t_bytes, t_flops = sb / (peak * 1e9), fl / (tpk * 1e12)
+    lm_flops = 2 * wl.T * wl.hidden_dim * wl.vocab
+    if lm_flops / lmb <= (tpk * 1e12) / (peak * 1e9):
+        lm_roofline = {"kernel": "lmhead_tc_kernel", "bound": "hbm", "achieved": achieved,
+                       "peak": peak, "unit": "GB/s", "frac": achieved / peak,
+                       "peak_source": peak_kind + " hbm_gbs (MEASURED_PEAKS.json)",
+                       "algorithmic_bytes_per_launch": lmb, "avg_launch_us": 1e3 * lm_ms,
+                       "traffic": LMHEAD_TRAFFIC_BYTES if CONFIG == 2 and packed else None}
+    else:
+        tf = lm_flops / (lm_ms * 1e-3) / 1e12
+        lm_roofline = {"kernel": "lmhead_tc_kernel", "bound": "tensor", "achieved": tf,
+                       "peak": tpk, "unit": "TFLOP/s", "frac": tf / tpk,
+                       "peak_source": tpk_kind + " bf16_tflops (MEASURED_PEAKS.json)",
+                       "algorithmic_flops_per_launch": lm_flops, "avg_launch_us": 1e3 * lm_ms,
+                       "traffic": None}
     line = {
         "metric": METRIC, "value": job_value(wl.T, world, ms * 1e-3), "unit": UNIT, "n_gpus": world,
         "steps": K, "warmup": W, "ms_per_step": ms, "us_per_step": 1e3 * ms,
-        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "bf16" if is_bf16 else "f32",
         "data": "synthetic (seeded; Llama-3.1-8B-shaped tensors, random weights)",
         "config": workload_config(wl),
         "lm_head_weight": ("packed once at load by asd_pack_lm_head (same bytes, streaming order)"
                            if packed else "[vocab, hidden] rows"),
         "hbm_gbs": sb / (ms * 1e-3) / 1e9, "hbm_frac_of_" + peak_kind: sb / (ms * 1e-3) / 1e9 / peak,
-        "roofline": {"kernel": "lmhead_tc_kernel", "bound": "hbm", "achieved": achieved,
-                     "peak": peak, "unit": "GB/s", "frac": achieved / peak,
-                     "peak_source": peak_kind + " hbm_gbs (MEASURED_PEAKS.json)",
-                     "algorithmic_bytes_per_launch": lmb, "avg_launch_us": 1e3 * lm_ms,
-                     "traffic": LMHEAD_TRAFFIC_BYTES},
+        # the whole step against the binding resource: the time its bytes take at
+        # the measured copy bandwidth or its flops at the measured bf16 rate
+        "step_bound": {"binding": "hbm" if t_bytes >= t_flops else "tensor",
+                       "bytes": sb, "flops": fl, "t_bytes_us": 1e6 * t_bytes,
+                       "t_flops_us": 1e6 * t_flops,
+                       "frac": max(t_bytes, t_flops) / (ms * 1e-3),
+                       "peaks": f"{peak_kind} hbm_gbs {peak}, {tpk_kind} bf16_tflops {tpk}"},
+        "roofline": lm_roofline,
         "stages_us": {**{name: 1e3 * stage_ms[j] for j, name in enumerate(STAGES)},
                       "step_with_stage_events": 1e3 * staged_ms,
                       "note": "second timed region with events between kernels (no overlap)"},
@@ -418,7 +483,15 @@ def run_asd(args):
 
 
 def main():
+    global CONFIG, TAU
     args = parse()
+    from paper_2609_02897_gb300 import synth
+    if args.config not in synth.WORKLOADS:
+        raise SystemExit(f"unknown workload {args.config}")
+    if args.config != CONFIG:
+        args.no_cpu_baseline = True   # the oracle's full step is far too slow beyond the headline
+    CONFIG = args.config
+    TAU = args.tau if args.tau is not None else synth.WORKLOADS[CONFIG]["tau"][0]
     if args.impl == "reference":
         run_reference(args)
     else:

@@ -39,6 +39,20 @@ WORKLOADS = {
     5: dict(name="llama3.1-8b-paged-b64-ctx8192-tree128", dtype="bf16", B=64,
             ctx=(8192, 8192), Hq=32, Hkv=8, D=128, hidden=4096, vocab=128256,
             tree=("grown", 128, 12, 16), tau=(1.0, 0.5, 0.3, 0.1), page_size=16),
+    # The draft trees the paper itself verifies (Sec. 3.3, Sec. 4.1 and its
+    # configuration table), as (n_steps, top-k, ndt) with ndt counting the
+    # root: the deep chain (7,1,8), the wide end of the dynamic range (3,4,4),
+    # and EAGLE-3's static (3,1,4); margin threshold kappa = 0.2 as in the
+    # paper's main results, and 1.0 (strict verification).
+    6: dict(name="llama3.1-8b-b1-ctx2048-chain-7-1-8", dtype="bf16", B=1, ctx=(2048, 2048),
+            Hq=32, Hkv=8, D=128, hidden=4096, vocab=128256,
+            tree=("eagle", 7, 1, 8), tau=(0.2, 1.0), page_size=0),
+    7: dict(name="llama3.1-8b-b1-ctx2048-tree-3-4-4", dtype="bf16", B=1, ctx=(2048, 2048),
+            Hq=32, Hkv=8, D=128, hidden=4096, vocab=128256,
+            tree=("eagle", 3, 4, 4), tau=(0.2, 1.0), page_size=0),
+    8: dict(name="llama3.1-8b-b1-ctx2048-chain-3-1-4", dtype="bf16", B=1, ctx=(2048, 2048),
+            Hq=32, Hkv=8, D=128, hidden=4096, vocab=128256,
+            tree=("eagle", 3, 1, 4), tau=(0.2, 1.0), page_size=0),
 }
 
 # Reduced variants with the same structure (tree recipe, GQA group, paging,
@@ -50,6 +64,9 @@ SMALL = {
     3: dict(B=5, ctx=(40, 333), Hq=8, Hkv=2, hidden=384, vocab=3001),
     4: dict(B=2, ctx=(1100, 1100), Hq=8, Hkv=2, hidden=512, vocab=4999),
     5: dict(B=6, ctx=(200, 200), Hq=8, Hkv=2, hidden=512, vocab=5000),
+    6: dict(ctx=(300, 300), Hq=8, Hkv=2, hidden=512, vocab=5000),
+    7: dict(ctx=(300, 300), Hq=8, Hkv=2, hidden=512, vocab=5000),
+    8: dict(ctx=(300, 300), Hq=8, Hkv=2, hidden=512, vocab=5000),
 }
 
 P_TOP1 = 0.5      # drafted token = the target's top-1 of the parent row

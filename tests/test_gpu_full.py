@@ -13,7 +13,7 @@ from paper_2609_02897_gb300 import synth
 
 pytestmark = pytest.mark.gpu
 
-SAMPLED = {1: None, 2: None, 3: [0, 7, 15], 4: [0, 5], 5: [0, 41]}
+SAMPLED = {1: None, 2: None, 3: [0, 7, 15], 4: [0, 5], 5: [0, 41], 6: None, 7: None, 8: None}
 
 
 @pytest.fixture(scope="module")
@@ -41,7 +41,7 @@ def _properties(wl, out):
     H.untouched_cache_equal(wl, out, written)
 
 
-@pytest.mark.parametrize("cfg", [1, 2, 3, 4, 5])
+@pytest.mark.parametrize("cfg", sorted(synth.WORKLOADS))
 def test_full_size(dev, cfg):
     wl = synth.make_workload(cfg)
     seqs = SAMPLED[cfg]

@@ -10,7 +10,7 @@ from paper_2609_02897_gb300 import synth
 
 pytestmark = pytest.mark.gpu
 
-CASES = [(cfg, tau) for cfg in (1, 2, 3, 4, 5) for tau in synth.WORKLOADS[cfg]["tau"]]
+CASES = [(cfg, tau) for cfg in sorted(synth.WORKLOADS) for tau in synth.WORKLOADS[cfg]["tau"]]
 
 
 @pytest.fixture(scope="module")

@@ -34,6 +34,27 @@ def test_eagle_tree_recipe():
         assert np.all(np.diff(d) >= 0)   # numbered by depth
 
 
+def test_paper_trees():
+    """The paper's (n_steps, top-k, ndt) shapes, ndt counting the root: the
+    top-1 triplets are chains of ndt nodes; (3, 4, 4) keeps 4 nodes of a
+    depth-3, 4-way expansion, ancestor-closed."""
+    rng = np.random.default_rng(5)
+    np.testing.assert_array_equal(synth.tree_eagle(rng, 7, 1, 8), [-1, 0, 1, 2, 3, 4, 5, 6])
+    np.testing.assert_array_equal(synth.tree_eagle(rng, 3, 1, 4), [-1, 0, 1, 2])
+    for _ in range(20):
+        p = synth.tree_eagle(rng, 3, 4, 4)
+        assert len(p) == 4 and p[0] == -1
+        _check_topo(p)
+        depth = [0] * 4
+        for i in range(1, 4):
+            depth[i] = depth[p[i]] + 1
+        assert max(depth) <= 3
+        assert max(np.bincount(p[1:], minlength=4)) <= 4
+    for cfg, shape in ((6, (7, 1, 8)), (7, (3, 4, 4)), (8, (3, 1, 4))):
+        assert synth.WORKLOADS[cfg]["tree"] == ("eagle",) + shape
+        assert 0.2 in synth.WORKLOADS[cfg]["tau"]
+
+
 def test_grown_tree_limits_and_spine():
     rng = np.random.default_rng(4)
     for n, dep, wid in [(64, 10, 10), (128, 12, 16), (96, 3, 1), (30, 5, 2)]:
@@ -53,7 +74,7 @@ def test_relabel_keeps_topological_order():
     assert sorted(np.bincount(q[1:], minlength=40)) == sorted(np.bincount(p[1:], minlength=40))
 
 
-@pytest.mark.parametrize("cfg", [1, 2, 3, 4, 5])
+@pytest.mark.parametrize("cfg", sorted(synth.WORKLOADS))
 def test_small_workloads_deterministic_and_consistent(cfg):
     a = synth.make_workload(cfg, small=True)
     b = synth.make_workload(cfg, small=True)
