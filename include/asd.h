@@ -12,7 +12,7 @@
  *      writing logits to memory, reduces every row to its max, argmax and
  *      log-sum-exp and evaluates the margin rule of Eq. 1 for every drafted
  *      token (asd_lmhead_margin);
- *   3. picks the longest root-to-node path of accepted nodes (asd_accept_path);
+ *   3. picks the committed root-to-node path of accepted nodes (asd_accept_path);
  *   4. appends the K/V of that path to the cache (asd_kv_compact).
  * asd_verify_step chains the four on one stream.
  *
@@ -53,7 +53,7 @@
 extern "C" {
 #endif
 
-#define ASD_ABI_VERSION 2
+#define ASD_ABI_VERSION 3
 #define ASD_MAX_TREE_NODES 128
 #define ASD_NUM_STAGE_EVENTS 5
 
@@ -71,6 +71,24 @@ typedef enum asd_status {
 } asd_status;
 
 typedef enum asd_dtype { ASD_F32 = 0, ASD_BF16 = 1 } asd_dtype;
+
+/* Which committed path a verify step picks (step 3).  The paper states the
+ * margin rule at the first mismatch position of a verification walk (Sec.
+ * 3.2); these are its readings on a tree ("promoted" = accepted by the margin
+ * rule but not the parent row's top-1):
+ *   LONGEST      the longest root-to-node path of accepted nodes (default);
+ *   ONCE         the longest one holding at most one promoted node;
+ *   GREEDY       from the root, a strict child if any (lowest index), else the
+ *                accepted child of largest ratio (lowest index on ties);
+ *   GREEDY_ONCE  the greedy walk with a single promotion.
+ * Equally long candidates are ordered by their node-index sequences, the
+ * smallest wins. */
+typedef enum asd_accept_rule {
+  ASD_ACCEPT_LONGEST = 0,
+  ASD_ACCEPT_ONCE = 1,
+  ASD_ACCEPT_GREEDY = 2,
+  ASD_ACCEPT_GREEDY_ONCE = 3
+} asd_accept_rule;
 
 /* Layout of the LM-head weight passed as w_lm. */
 typedef enum asd_lm_layout {
@@ -96,6 +114,7 @@ typedef struct asd_dims {
   int32_t max_path;     /* columns of the path output, >= longest root-to-leaf
                            path (nodes, root included)                         */
   int32_t lm_head_layout; /* asd_lm_layout of w_lm                             */
+  int32_t accept_rule;    /* asd_accept_rule of step 3                          */
 } asd_dims;
 
 /* Bytes of device workspace that the calls below need for `total_nodes`
@@ -172,17 +191,20 @@ asd_status asd_pack_lm_head(const asd_dims* dims, const void* w, void* w_packed,
 /*
  * Accepted path (step 3; Sec. 3.2 and Fig. 1: verification commits the
  * drafted tokens up to the first node that is neither a strict match nor
- * promoted by the margin rule).  Over the tree this is the longest root-to-
- * node path whose non-root nodes all have accept = 1; equally long paths are
- * ordered by their node-index sequences and the smallest wins.
+ * promoted by the margin rule).  Over the tree: the path dims->accept_rule
+ * picks among root-to-node paths whose non-root nodes all have accept = 1
+ * (by default the longest, equally long paths ordered by their node-index
+ * sequences, the smallest winning).
  *  accept [T] uint8, row_argmax [T] int32, tokens [T] int32 (inputs)
+ *  ratio [T] float (Eq. 1, as asd_lmhead_margin writes it): read by the
+ *  greedy rules only, may be NULL for the others
  *  path [B, max_path] int32: local node ids, root first, -1 padded
  *  path_len [B]: nodes on the path including the root (>= 1)
  *  bonus [B]: row_argmax of the last path node (the next committed token)
  *  n_promoted [B]: path nodes whose token is not the parent row's argmax
  */
 asd_status asd_accept_path(const asd_dims* dims, const int32_t* parent, const int32_t* tokens,
-                           const uint8_t* accept, const int32_t* row_argmax,
+                           const uint8_t* accept, const int32_t* row_argmax, const float* ratio,
                            const int32_t* cu_nodes, int32_t total_nodes, int32_t* path,
                            int32_t* path_len, int32_t* bonus, int32_t* n_promoted,
                            void* workspace, size_t workspace_bytes, void* stream);

@@ -21,6 +21,7 @@ _lib = ctypes.CDLL(_LIB_PATH)
 
 ASD_F32, ASD_BF16 = 0, 1
 ASD_LM_ROWS, ASD_LM_PACKED = 0, 1
+ASD_ACCEPT_LONGEST, ASD_ACCEPT_ONCE, ASD_ACCEPT_GREEDY, ASD_ACCEPT_GREEDY_ONCE = 0, 1, 2, 3
 MAX_TREE_NODES = 128
 NUM_STAGE_EVENTS = 5
 STATUS = {0: "ASD_OK", 1: "ASD_ERR_INVALID_ARG", 2: "ASD_ERR_SHAPE", 3: "ASD_ERR_TREE",
@@ -42,7 +43,8 @@ class AsdError(RuntimeError):
 class Dims(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int32) for n in (
         "batch", "num_q_heads", "num_kv_heads", "head_dim", "hidden", "vocab", "dtype",
-        "page_size", "ctx_max", "num_pages", "max_nodes", "max_path", "lm_head_layout")]
+        "page_size", "ctx_max", "num_pages", "max_nodes", "max_path", "lm_head_layout",
+        "accept_rule")]
 
 
 _vp = ctypes.c_void_p
@@ -74,7 +76,7 @@ _lib.asd_lmhead_margin.restype = ctypes.c_int
 _lib.asd_lmhead_margin.argtypes = [_P] + [_vp] * 5 + [ctypes.c_int32, ctypes.c_float] + [_vp] * 6 + [
     _vp, ctypes.c_size_t, _vp]
 _lib.asd_accept_path.restype = ctypes.c_int
-_lib.asd_accept_path.argtypes = [_P] + [_vp] * 5 + [ctypes.c_int32] + [_vp] * 4 + [
+_lib.asd_accept_path.argtypes = [_P] + [_vp] * 6 + [ctypes.c_int32] + [_vp] * 4 + [
     _vp, ctypes.c_size_t, _vp]
 _lib.asd_kv_compact.restype = ctypes.c_int
 _lib.asd_kv_compact.argtypes = [_P, _vp, _vp, _vp, ctypes.c_int32] + [_vp] * 7 + [
@@ -101,9 +103,9 @@ def abi_version() -> int:
 
 
 def make_dims(batch, num_q_heads, num_kv_heads, head_dim, hidden, vocab, dtype, page_size,
-              ctx_max, num_pages, max_nodes, max_path, lm_head_layout=0) -> Dims:
+              ctx_max, num_pages, max_nodes, max_path, lm_head_layout=0, accept_rule=0) -> Dims:
     return Dims(batch, num_q_heads, num_kv_heads, head_dim, hidden, vocab, dtype, page_size,
-                ctx_max, num_pages, max_nodes, max_path, lm_head_layout)
+                ctx_max, num_pages, max_nodes, max_path, lm_head_layout, accept_rule)
 
 
 def _ptr(t: Optional[torch.Tensor]):
@@ -190,10 +192,10 @@ def asd_lmhead_margin_noalloc(dims, hidden, w_lm, tokens, parent, cu_nodes, tau,
 
 
 def asd_accept_path(dims, parent, tokens, accept, row_argmax, cu_nodes, path, path_len, bonus,
-                    n_promoted, workspace, stream=None):
+                    n_promoted, workspace, stream=None, ratio=None):
     _check(_lib.asd_accept_path(
         ctypes.byref(dims), _ptr(parent), _ptr(tokens), _ptr(accept), _ptr(row_argmax),
-        _ptr(cu_nodes), int(parent.numel()), _ptr(path), _ptr(path_len), _ptr(bonus),
+        _ptr(ratio), _ptr(cu_nodes), int(parent.numel()), _ptr(path), _ptr(path_len), _ptr(bonus),
         _ptr(n_promoted), _ptr(workspace), workspace.numel(), _stream(stream)),
         "asd_accept_path")
 

@@ -88,6 +88,7 @@ bool dims_ok(const asd_dims* d) {
   if (d->max_path < 1) return false;
   if (d->lm_head_layout != ASD_LM_ROWS && d->lm_head_layout != ASD_LM_PACKED) return false;
   if (d->lm_head_layout == ASD_LM_PACKED && d->dtype != ASD_BF16) return false;
+  if (d->accept_rule < ASD_ACCEPT_LONGEST || d->accept_rule > ASD_ACCEPT_GREEDY_ONCE) return false;
   return true;
 }
 
@@ -275,6 +276,7 @@ asd_status run_lmhead(const Ctx& c, const void* hidden, const void* w, float* l_
 TailParams tail_params(const Ctx& c, int mode) {
   TailParams t{};
   t.mode = mode;
+  t.rule = c.d.accept_rule;
   t.part = ws_at<LmPartial>(c.ws, c.L.lm_part);
   t.g_lm = c.L.g_lm;
   t.status = ws_at<int>(c.ws, c.L.status);
@@ -410,17 +412,19 @@ asd_status asd_lmhead_margin(const asd_dims* dims, const void* hidden, const voi
 }
 
 asd_status asd_accept_path(const asd_dims* dims, const int32_t* parent, const int32_t* tokens,
-                           const uint8_t* accept, const int32_t* row_argmax,
+                           const uint8_t* accept, const int32_t* row_argmax, const float* ratio,
                            const int32_t* cu_nodes, int32_t total_nodes, int32_t* path,
                            int32_t* path_len, int32_t* bonus, int32_t* n_promoted,
                            void* workspace, size_t workspace_bytes, void* stream) {
   if (!parent || !tokens || !accept || !row_argmax || !cu_nodes || !path || !path_len || !bonus ||
       !n_promoted)
     return ASD_ERR_INVALID_ARG;
+  if (dims && dims->accept_rule >= ASD_ACCEPT_GREEDY && !ratio) return ASD_ERR_INVALID_ARG;
   Ctx c;
   asd_status st = begin_call(dims, total_nodes, workspace, workspace_bytes, stream, &c);
   if (st != ASD_OK) return st;
   TailParams t = tail_params(c, kTailWalk);
+  t.ratio = const_cast<float*>(ratio);
   t.parent = parent;
   t.tokens = tokens;
   t.cu_nodes = cu_nodes;

@@ -158,7 +158,7 @@ struct TailParams {
   int32_t* row_argmax;        // written by finalize, read by walk
   float* row_lse;
   const float* l_draft;
-  float* ratio;
+  float* ratio;               // written by finalize; read by the greedy walks otherwise
   uint8_t* accept;            // written by finalize, read by walk
   // walk
   int32_t* path;              // [B, max_path]
@@ -174,6 +174,7 @@ struct TailParams {
   const int32_t* page_table;
   int32_t* ctx_len_out;
   int* status;
+  int rule;                   // accepted-path reading (asd_accept_rule)
   int B, T, Hkv, D, elem_bytes, max_nodes, max_path;
   int ctx_max, page_size, pages_per_seq, num_pages;
 };

@@ -5,10 +5,17 @@
 //            every drafted node: ratio = exp(l_draft - row_max[parent]) (Eq. 1),
 //            accept = strict match of the parent row's top-1 or ratio >= tau
 //            (compared as l_draft - row_max >= ln tau);
-//  walk      choose the longest root-to-node path of accepted nodes, ties to the
-//            lexicographically smallest node sequence (Sec. 3.2): heights of
-//            accepted subtrees bottom-up by depth, then from the root follow
-//            the lowest-index accepted child whose height is one less;
+//  walk      choose the committed path under one of four readings of the
+//            paper's first-mismatch rule (Sec. 3.2; TailParams::rule):
+//            0 the longest root-to-node path of accepted nodes, ties to the
+//              lexicographically smallest node sequence: heights of accepted
+//              subtrees bottom-up by depth, then from the root the
+//              lowest-index accepted child whose height is one less;
+//            1 the same over paths with at most one promoted node (accepted,
+//              not a strict match): strict-only and one-promotion heights;
+//            2 greedy: a strict child if any (lowest index), else the accepted
+//              child of largest ratio (lowest index on ties), else stop;
+//            3 greedy with a single promotion;
 //  compact   copy the path's tree K/V into cache slots ctx_len .. ctx_len +
 //            path_len - 1 (contiguous or through the page table).
 #include <climits>
@@ -47,6 +54,10 @@ __global__ void __launch_bounds__(kTailThreads) tail_kernel(const TailParams p) 
   __shared__ int s_h[kMaxNodes];
   __shared__ int s_bc[kMaxNodes];
   __shared__ int s_path[kMaxNodes];
+  __shared__ int s_h1[kMaxNodes];                    // rule 1: heights with one promotion
+  __shared__ int s_bc1[kMaxNodes];                   // rule 1: best child, promotion left
+  __shared__ float s_ratio[kMaxNodes];               // rules 2, 3
+  __shared__ unsigned long long s_bp[kMaxNodes];     // rules 2, 3: best promoted child key
   __shared__ int s_maxd, s_len, s_skip;
 
   // Until pdl_wait() this kernel reads only caller inputs (cu_nodes, parent,
@@ -96,6 +107,9 @@ __global__ void __launch_bounds__(kTailThreads) tail_kernel(const TailParams p) 
     s_dep[i] = d;
     s_h[i] = 1;
     s_bc[i] = INT_MAX;
+    s_h1[i] = 1;
+    s_bc1[i] = INT_MAX;
+    s_bp[i] = 0ull;
     atomicMax(&s_maxd, d);
   }
 
@@ -156,11 +170,13 @@ __global__ void __launch_bounds__(kTailThreads) tail_kernel(const TailParams p) 
       p.ratio[s + i] = ratio;
       p.accept[s + i] = static_cast<uint8_t>(acc);
       s_acc[i] = acc;
+      s_ratio[i] = ratio;
     }
   } else if (p.mode & kTailWalk) {
     if (i < n) {
       s_acc[i] = p.accept[s + i] != 0 ? 1 : 0;
       s_arg[i] = p.row_argmax[s + i];
+      s_ratio[i] = (p.rule >= 2 && p.ratio) ? p.ratio[s + i] : 0.f;
     }
   }
   __syncthreads();
@@ -168,18 +184,56 @@ __global__ void __launch_bounds__(kTailThreads) tail_kernel(const TailParams p) 
   // -------------------------------------------------------------------- walk
   if (p.mode & kTailWalk) {
     if (!s_skip) {
-      for (int dd = s_maxd; dd >= 1; --dd) {
-        if (i < n && s_dep[i] == dd && s_acc[i]) atomicMax(&s_h[s_par[i]], s_h[i] + 1);
-        __syncthreads();
+      // a node is strict when it drafts its parent row's top-1; root-level
+      // quantities are per node below, the walk runs on thread 0
+      const bool strict_i = i > 0 && i < n && s_acc[i] && s_tok[i] == s_arg[s_par[i]];
+      if (p.rule <= 1) {
+        // s_h: heights over accepted (rule 0) or strict-only (rule 1) children;
+        // s_h1: heights with at most one promotion below the node (rule 1)
+        for (int dd = s_maxd; dd >= 1; --dd) {
+          if (i < n && s_dep[i] == dd && s_acc[i]) {
+            if (p.rule == 0 || strict_i) atomicMax(&s_h[s_par[i]], s_h[i] + 1);
+            if (p.rule == 1) atomicMax(&s_h1[s_par[i]], (strict_i ? s_h1[i] : s_h[i]) + 1);
+          }
+          __syncthreads();
+        }
+        if (i > 0 && i < n && s_acc[i]) {
+          const int u = s_par[i];
+          if ((p.rule == 0 || strict_i) && s_h[i] == s_h[u] - 1) atomicMin(&s_bc[u], i);
+          if (p.rule == 1 && (strict_i ? s_h1[i] : s_h[i]) == s_h1[u] - 1) atomicMin(&s_bc1[u], i);
+        }
+      } else if (i > 0 && i < n && s_acc[i]) {
+        const int u = s_par[i];
+        if (strict_i) {
+          atomicMin(&s_bc[u], i);
+        } else {
+          // largest ratio first, then the lowest index (ratios are >= 0 here)
+          const unsigned long long key =
+              (static_cast<unsigned long long>(__float_as_uint(fmaxf(s_ratio[i], 0.f))) << 32) |
+              static_cast<unsigned long long>(0xFFFFFFFFu - static_cast<unsigned>(i));
+          atomicMax(&s_bp[u], key);
+        }
       }
-      if (i > 0 && i < n && s_acc[i] && s_h[i] == s_h[s_par[i]] - 1) atomicMin(&s_bc[s_par[i]], i);
       __syncthreads();
       if (i == 0) {
-        int u = 0, len = 0, promoted = 0;
+        int u = 0, len = 0, promoted = 0, budget = 1;
         s_path[len++] = 0;
-        while (s_bc[u] != INT_MAX && len < kMaxNodes) {
-          const int c = s_bc[u];
-          if (s_tok[c] != s_arg[u]) ++promoted;
+        while (len < kMaxNodes) {
+          int c = INT_MAX;
+          if (p.rule == 0) {
+            c = s_bc[u];
+          } else if (p.rule == 1) {
+            c = budget ? s_bc1[u] : s_bc[u];
+          } else {
+            c = s_bc[u];
+            if (c == INT_MAX && s_bp[u] != 0ull && (p.rule == 2 || budget))
+              c = static_cast<int>(0xFFFFFFFFu - static_cast<unsigned>(s_bp[u] & 0xFFFFFFFFull));
+          }
+          if (c == INT_MAX) break;
+          if (s_tok[c] != s_arg[u]) {
+            ++promoted;
+            budget = 0;
+          }
           s_path[len++] = c;
           u = c;
         }

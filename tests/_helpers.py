@@ -114,9 +114,10 @@ def valid_path(parent_local, accept_local, path):
     return len(path) == best
 
 
-def compare_verify(wl, tau, out, seqs=None, check_attn_nodes=None):
+def compare_verify(wl, tau, out, seqs=None, check_attn_nodes=None, rule=0):
     """Compares one verify step's outputs (numpy copies in `out`) with the
-    oracle on the sequences `seqs` (all by default).  Returns a Report."""
+    oracle on the sequences `seqs` (all by default), the committed path under
+    accepted-path reading `rule`.  Returns a Report."""
     rep = Report()
     atol, rtol = tol(wl)
     B = wl.B
@@ -162,6 +163,14 @@ def compare_verify(wl, tau, out, seqs=None, check_attn_nodes=None):
             continue
         assert out["accept"][c] == lm["accept"][c], \
             f"accept node {c}: gpu {out['accept'][c]} oracle {lm['accept'][c]} ratio {lm['ratio'][c]}"
+    if rule >= 2:
+        # the greedy walks order promoted siblings by ratio: near-equal ratios
+        # cannot be ordered alike in fp32 and fp64
+        for u in nodes:
+            sib = sorted((float(lm["ratio"][c]) for c in kids if gp[c] == u and lm["accept"][c]
+                          and int(wl.tokens[c]) != int(lm["row_argmax"][u])), reverse=True)
+            if len(sib) > 1 and sib[0] - sib[1] < 1e-3:
+                band.update(int(c) for c in kids if gp[c] == u)
     rep.band_nodes = len(band)
 
     # steps 3-4: path and commit
@@ -171,13 +180,19 @@ def compare_verify(wl, tau, out, seqs=None, check_attn_nodes=None):
         path = [int(x) for x in out["path"][b][:plen]]
         assert all(int(x) == -1 for x in out["path"][b][plen:])
         acc_gpu = out["accept"][s:e]
-        assert valid_path(list(wl.parent[s:e]), list(acc_gpu), path), f"seq {b} path {path}"
+        if rule == 0:
+            assert valid_path(list(wl.parent[s:e]), list(acc_gpu), path), f"seq {b} path {path}"
+        # the walk itself, on the GPU's own verdicts, is exact
+        own = oracle.accept_path(wl.parent[s:e], acc_gpu, out["row_argmax"][s:e], wl.tokens[s:e],
+                                 [0, e - s], rule=rule, ratio=out["ratio"][s:e])
+        assert path == own[0][0], f"seq {b} rule {rule}: gpu {path} walk on its verdicts {own[0][0]}"
         if band.intersection(range(s, e)):
             rep.excluded_seqs += 1
         else:
             rep.checked_seqs += 1
             paths, plens, bonus, npro = oracle.accept_path(
-                wl.parent[s:e], lm["accept"][s:e], lm["row_argmax"][s:e], wl.tokens[s:e], [0, e - s])
+                wl.parent[s:e], lm["accept"][s:e], lm["row_argmax"][s:e], wl.tokens[s:e], [0, e - s],
+                rule=rule, ratio=lm["ratio"][s:e])
             assert path == paths[0], f"seq {b}: gpu {path} oracle {paths[0]}"
             assert int(out["bonus"][b]) == int(bonus[0])
             assert int(out["n_promoted"][b]) == int(npro[0])

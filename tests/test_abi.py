@@ -34,7 +34,7 @@ def test_binding_names_match_header():
     build.build()
     from paper_2609_02897_gb300 import asd
     assert sorted(asd.EXPORTS) == _declared()
-    assert asd.abi_version() == 2
+    assert asd.abi_version() == 3
 
 
 def test_host_checks_without_gpu(lib):
@@ -75,3 +75,25 @@ def test_packed_lm_head_host_checks(lib):
     assert fn(ctypes.byref(d), w, ctypes.c_void_p((1 << 30) + 16), 1 << 30, None) == 1  # alignment
     assert fn(ctypes.byref(d), w, out, 4096, None) == 6                                 # too small
     assert fn(ctypes.byref(d), w, ctypes.c_void_p((1 << 20) + 256), 1 << 30, None) == 1  # overlap
+
+
+def test_accept_rule_host_checks(lib):
+    """An accept rule outside asd_accept_rule fails the dims check
+    (ASD_ERR_SHAPE) and the greedy rules need the ratios
+    (ASD_ERR_INVALID_ARG without them); both are answered before any CUDA
+    call, so the placeholder pointers are never read."""
+    from paper_2609_02897_gb300 import asd
+    d = asd.make_dims(1, 4, 4, 64, 256, 4096, asd.ASD_BF16, 0, 64, 0, 8, 5)
+    fn = asd._lib.asd_accept_path
+    buf = ctypes.c_void_p(1 << 20)
+
+    def call(ratio):
+        return fn(ctypes.byref(d), buf, buf, buf, buf, ratio, buf, 8, buf, buf, buf, buf, buf,
+                  1 << 20, None)
+    for rule in (-1, 4):
+        d.accept_rule = rule
+        assert call(buf) == 2
+        assert lib.asd_workspace_bytes(ctypes.byref(d), 8) == 0
+    for rule in (asd.ASD_ACCEPT_GREEDY, asd.ASD_ACCEPT_GREEDY_ONCE):
+        d.accept_rule = rule
+        assert call(None) == 1

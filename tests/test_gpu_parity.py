@@ -240,3 +240,52 @@ def test_cuda_graph_replay_matches_eager(dev):
     for k, v in step.out.items():
         got = v.float().cpu().numpy() if v.is_floating_point() else v.cpu().numpy()
         np.testing.assert_array_equal(got, eager[k], err_msg=k)
+
+
+@pytest.mark.parametrize("rule", [1, 2, 3])
+@pytest.mark.parametrize("cfg,tau", [(2, 0.3), (3, 0.5), (5, 0.1), (6, 0.2), (7, 0.2)])
+def test_accept_rules(dev, cfg, tau, rule):
+    """The other readings of the first-mismatch rule (asd_accept_rule) against
+    the oracle's literal enumeration / walk."""
+    wl = H.prepared(cfg, small=True)
+    out, status, _, _ = dev.run_verify(wl, tau, rule=rule)
+    assert status == 0
+    rep = H.compare_verify(wl, tau, out, rule=rule)
+    H.untouched_cache_equal(wl, out, _written(wl, out))
+    if rule in (1, 3):
+        assert np.all(out["n_promoted"] <= 1)
+    print(wl.name, tau, rule, rep)
+
+
+@pytest.mark.parametrize("rule", [2, 3])
+def test_greedy_accept_path_call_matches_verify_step(dev, rule):
+    """asd_accept_path with the ratios asd_lmhead_margin wrote gives the verify
+    step's path."""
+    import torch
+    from paper_2609_02897_gb300 import asd
+    wl = H.prepared(3, small=True)
+    ref, status, _, _ = dev.run_verify(wl, 0.1, rule=rule)
+    assert status == 0
+    d = dev.to_device(wl)
+    dims = dev.dims_of(wl)
+    dims.accept_rule = rule
+    T, B = wl.T, wl.B
+    ws = asd.alloc_workspace(dims, T)
+    f = lambda: torch.empty(T, dtype=torch.float32, device="cuda")  # noqa: E731
+    i = lambda n: torch.empty(n, dtype=torch.int32, device="cuda")  # noqa: E731
+    rm, ra, rl, ld, rt = f(), i(T), f(), f(), f()
+    acc = torch.empty(T, dtype=torch.uint8, device="cuda")
+    asd.asd_lmhead_margin(dims, d["hidden"], d["w_lm"], d["tokens"], d["parent"], d["cu_nodes"], 0.1,
+                          rm, ra, rl, ld, rt, acc, ws)
+    path = torch.empty(B, dims.max_path, dtype=torch.int32, device="cuda")
+    plen, bonus, npro = i(B), i(B), i(B)
+    asd.asd_accept_path(dims, d["parent"], d["tokens"], acc, ra, d["cu_nodes"], path, plen, bonus,
+                        npro, ws, ratio=rt)
+    torch.cuda.synchronize()
+    assert asd.asd_get_device_status(ws) == 0
+    for name, t in [("path", path), ("path_len", plen), ("bonus", bonus), ("n_promoted", npro)]:
+        np.testing.assert_array_equal(t.cpu().numpy(), ref[name], err_msg=name)
+    with pytest.raises(asd.AsdError) as e:   # the greedy rules read the ratios
+        asd.asd_accept_path(dims, d["parent"], d["tokens"], acc, ra, d["cu_nodes"], path, plen,
+                            bonus, npro, ws)
+    assert e.value.code == 1
