@@ -16,9 +16,12 @@ Modules
   accept     longest accepted root-to-node path by literal enumeration (a3)
   compact    copy of the accepted nodes' K/V into the cache (a4)
   verify     the four steps chained
+  policy     the dynamic tree-shape policy: DCS, RAR, triplet mapping and
+             circuit breaker (Sec. 3.3, Eq. 2)
 """
 from .attention import tree_attention, ancestors_of  # noqa: F401
 from .lmhead import logits_rows, lmhead_margin, topk_tokens  # noqa: F401
 from .accept import accept_path  # noqa: F401
 from .compact import kv_compact  # noqa: F401
 from .verify import verify_step  # noqa: F401
+from . import policy  # noqa: F401
