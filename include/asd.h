@@ -53,7 +53,7 @@
 extern "C" {
 #endif
 
-#define ASD_ABI_VERSION 3
+#define ASD_ABI_VERSION 4
 #define ASD_MAX_TREE_NODES 128
 #define ASD_NUM_STAGE_EVENTS 5
 
@@ -306,6 +306,82 @@ asd_status asd_lmhead_margin_noalloc(const asd_dims* dims, const void* hidden, c
                                      float* row_max, int32_t* row_argmax, float* row_lse,
                                      float* l_draft, float* ratio, uint8_t* accept,
                                      int32_t* device_status, void* stream);
+
+/*
+ * Dynamic tree-shape policy (Sec. 3.3, Eq. 2).  Per request, once per
+ * decoding step, the Draft Confidence Score
+ *     DCS = min(1, p_draft(top1) * RAR / divisor)
+ * maps linearly onto a range of draft-tree triplets (n_steps, topk, ndt):
+ * n_steps and ndt move from `shallow` (DCS = 0) to `deep` (DCS = 1) with DCS,
+ * topk with 1 - DCS; each coordinate is start + round(span * u) with the
+ * product in binary64 and halves rounded upward.  RAR is an exponential
+ * moving average of the fraction of drafted nodes the target accepted:
+ *     RAR <- alpha * (path_len - 1) / (nodes - 1) + (1 - alpha) * RAR,
+ * starting at rar_init; the DCS of a step uses the RAR after the previous
+ * step's verification.  A request with `breaker` consecutive verify steps that
+ * accepted no drafted node returns to its starting state (RAR = rar_init).
+ * Steps that verified only the root, or whose sequence was rejected
+ * (path_len 0), leave the state unchanged.  All arithmetic is binary64 with
+ * every product and sum rounded on its own (no fused multiply-add), so the
+ * results do not depend on the compiler.
+ * The paper's settings: alpha 0.3, divisor 0.5, shallow (3, 4, 4), deep
+ * (7, 1, 8), breaker 5.
+ */
+typedef struct asd_policy_params {
+  double alpha;       /* EMA weight of the newest step, in (0, 1]                */
+  double divisor;     /* d > 0                                                    */
+  double rar_init;    /* RAR at the start and after a breaker reset, in [0, 1]    */
+  int32_t shallow[3]; /* (n_steps, topk, ndt) at DCS = 0; each in [1, 128]        */
+  int32_t deep[3];    /* (n_steps, topk, ndt) at DCS = 1; each in [1, 128]        */
+  int32_t breaker;    /* consecutive zero-accept steps that reset a request, >= 1 */
+  int32_t reserved;   /* must be 0                                                */
+} asd_policy_params;
+
+/* Per-request policy state, an array of `batch` of these in device memory
+ * (16 bytes each, 8-byte aligned), owned by the caller. */
+typedef struct asd_policy_state {
+  double rar;          /* running acceptance rate                          */
+  int32_t zero_streak; /* consecutive steps without an accepted draft      */
+  int32_t breaks;      /* circuit-breaker resets so far                    */
+} asd_policy_state;
+
+/* Host only (no CUDA call): every triplet the mapping returns for some DCS in
+ * [0, 1], in the order of increasing DCS, so that a caller can capture one
+ * CUDA graph per triplet ahead of time (Sec. 3.3).  Writes min(count, cap)
+ * triplets to out[3 * i + {0, 1, 2}] (out may be NULL when cap is 0) and
+ * returns their count, or -ASD_ERR_INVALID_ARG for invalid params. */
+int32_t asd_policy_triplets(const asd_policy_params* params, int32_t* out, int32_t cap);
+
+/* Sets every request's state to its start (RAR = rar_init, counts 0).
+ * state: device array [batch].  Enqueued on `stream`; batch 0 enqueues
+ * nothing.  Errors: null pointers, invalid params or batch < 0 ->
+ * ASD_ERR_INVALID_ARG; launch failure -> ASD_ERR_CUDA. */
+asd_status asd_policy_init(const asd_policy_params* params, asd_policy_state* state,
+                           int32_t batch, void* stream);
+
+/* Folds one verify step into each request's state: request b verified
+ * cu_nodes[b+1] - cu_nodes[b] nodes (root included) and committed path_len[b]
+ * of them (root included), as written by asd_accept_path or
+ * asd_verify_step.  cu_nodes [batch+1], path_len [batch]: device int32.  A
+ * request whose counts are inconsistent (path_len outside [0, nodes]) is left
+ * unchanged.  Errors as asd_policy_init. */
+asd_status asd_policy_update(const asd_policy_params* params, const int32_t* cu_nodes,
+                             const int32_t* path_len, int32_t batch, asd_policy_state* state,
+                             void* stream);
+
+/* Picks each request's next triplet.  p_draft(top1) of request b is
+ * exp(row_max[r] - row_lse[r]) of the draft model's LM-head row r = rows[b]
+ * (rows may be NULL: r = b), i.e. the row statistics asd_lmhead_margin
+ * writes when run on the draft's LM head.  row_max, row_lse: device float
+ * [num_rows].  Writes triplet[3 * b + {0, 1, 2}] = (n_steps, topk, ndt)
+ * (device int32 [batch][3]) and, if dcs is not NULL, dcs[b] (device double).
+ * The state is only read.  A row index outside [0, num_rows) gives the
+ * triplet (0, 0, 0) and DCS NaN for that request; a probability that is not
+ * a number counts as 0.  Errors as asd_policy_init. */
+asd_status asd_policy_select(const asd_policy_params* params, const float* row_max,
+                             const float* row_lse, const int32_t* rows, int32_t num_rows,
+                             int32_t batch, const asd_policy_state* state, int32_t* triplet,
+                             double* dcs, void* stream);
 
 #ifdef __cplusplus
 }

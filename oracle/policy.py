@@ -34,7 +34,10 @@ def p_top1(row_max, row_lse):
 
 def dcs(p, rar, divisor):
     """Eq. 2 rescaled by the divisor d and saturated at 1 (Sec. 3.3)."""
-    return min(1.0, (float(p) * float(rar)) / float(divisor))
+    p = float(p)
+    if not p >= 0.0:                     # a probability that is not a number counts as 0
+        p = 0.0
+    return min(1.0, (p * float(rar)) / float(divisor))
 
 
 def round_half_up(y):
@@ -113,7 +116,7 @@ def update(state, n_nodes, path_len, alpha, breaker, rar_init=1.0):
     """One verify step's effect on a request's policy state (Sec. 3.3):
     the EMA of the accepted fraction, then the circuit breaker."""
     n_nodes, path_len = int(n_nodes), int(path_len)
-    if n_nodes <= 1 or path_len <= 0:
+    if n_nodes <= 1 or path_len <= 0 or path_len > n_nodes:
         return state
     accepted = path_len - 1
     a = accepted / (n_nodes - 1)

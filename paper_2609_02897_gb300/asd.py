@@ -30,7 +30,8 @@ STATUS = {0: "ASD_OK", 1: "ASD_ERR_INVALID_ARG", 2: "ASD_ERR_SHAPE", 3: "ASD_ERR
 EXPORTS = ["asd_workspace_bytes", "asd_tree_attention", "asd_lmhead_margin", "asd_accept_path",
            "asd_kv_compact", "asd_verify_step", "asd_get_device_status", "asd_status_string",
            "asd_abi_version", "asd_lmhead_margin_noalloc", "asd_lm_head_packed_bytes",
-           "asd_pack_lm_head"]
+           "asd_pack_lm_head",
+           "asd_policy_triplets", "asd_policy_init", "asd_policy_update", "asd_policy_select"]
 
 
 class AsdError(RuntimeError):
@@ -64,7 +65,26 @@ class VerifyArgs(ctypes.Structure):
     ]
 
 
+class PolicyParams(ctypes.Structure):
+    """asd_policy_params: the tree-shape policy's settings (Sec. 3.3)."""
+    _fields_ = [("alpha", ctypes.c_double), ("divisor", ctypes.c_double),
+                ("rar_init", ctypes.c_double), ("shallow", ctypes.c_int32 * 3),
+                ("deep", ctypes.c_int32 * 3), ("breaker", ctypes.c_int32),
+                ("reserved", ctypes.c_int32)]
+
+
+POLICY_STATE_BYTES = 16
+
+
+def make_policy_params(alpha=0.3, divisor=0.5, rar_init=1.0, shallow=(3, 4, 4), deep=(7, 1, 8),
+                       breaker=5) -> PolicyParams:
+    """Defaults: the paper's settings (Sec. 3.3, Sec. 4.2)."""
+    return PolicyParams(alpha, divisor, rar_init, (ctypes.c_int32 * 3)(*shallow),
+                        (ctypes.c_int32 * 3)(*deep), breaker, 0)
+
+
 _P = ctypes.POINTER(Dims)
+_PP = ctypes.POINTER(PolicyParams)
 _lib.asd_abi_version.restype = ctypes.c_int32
 _lib.asd_status_string.restype = ctypes.c_char_p
 _lib.asd_status_string.argtypes = [ctypes.c_int32]
@@ -92,6 +112,15 @@ _lib.asd_lm_head_packed_bytes.restype = ctypes.c_size_t
 _lib.asd_lm_head_packed_bytes.argtypes = [_P]
 _lib.asd_pack_lm_head.restype = ctypes.c_int
 _lib.asd_pack_lm_head.argtypes = [_P, _vp, _vp, ctypes.c_size_t, _vp]
+_lib.asd_policy_triplets.restype = ctypes.c_int32
+_lib.asd_policy_triplets.argtypes = [_PP, _vp, ctypes.c_int32]
+_lib.asd_policy_init.restype = ctypes.c_int
+_lib.asd_policy_init.argtypes = [_PP, _vp, ctypes.c_int32, _vp]
+_lib.asd_policy_update.restype = ctypes.c_int
+_lib.asd_policy_update.argtypes = [_PP, _vp, _vp, ctypes.c_int32, _vp, _vp]
+_lib.asd_policy_select.restype = ctypes.c_int
+_lib.asd_policy_select.argtypes = [_PP, _vp, _vp, _vp, ctypes.c_int32, ctypes.c_int32, _vp, _vp,
+                                   _vp, _vp]
 
 
 def lib_path() -> str:
@@ -274,3 +303,74 @@ class VerifyStep:
 
     def device_status(self, stream=None) -> int:
         return asd_get_device_status(self.workspace, stream)
+
+
+# ------------------------------------------------------------ tree-shape policy
+
+def asd_policy_triplets(params: PolicyParams) -> list:
+    """Every (n_steps, topk, ndt) the policy can select, by increasing DCS
+    (host only)."""
+    n = int(_lib.asd_policy_triplets(ctypes.byref(params), None, 0))
+    if n < 0:
+        raise AsdError(-n, "asd_policy_triplets")
+    buf = (ctypes.c_int32 * (3 * n))()
+    _lib.asd_policy_triplets(ctypes.byref(params), buf, n)
+    return [tuple(buf[3 * i:3 * i + 3]) for i in range(n)]
+
+
+def asd_policy_init(params: PolicyParams, state: torch.Tensor, batch: int, stream=None):
+    _check(_lib.asd_policy_init(ctypes.byref(params), _ptr(state), int(batch), _stream(stream)),
+           "asd_policy_init")
+
+
+def asd_policy_update(params: PolicyParams, cu_nodes, path_len, batch: int, state, stream=None):
+    _check(_lib.asd_policy_update(ctypes.byref(params), _ptr(cu_nodes), _ptr(path_len),
+                                  int(batch), _ptr(state), _stream(stream)), "asd_policy_update")
+
+
+def asd_policy_select(params: PolicyParams, row_max, row_lse, rows, num_rows: int, batch: int,
+                      state, triplet, dcs=None, stream=None):
+    _check(_lib.asd_policy_select(ctypes.byref(params), _ptr(row_max), _ptr(row_lse), _ptr(rows),
+                                  int(num_rows), int(batch), _ptr(state), _ptr(triplet), _ptr(dcs),
+                                  _stream(stream)), "asd_policy_select")
+
+
+class TreePolicy:
+    """Per-request tree-shape policy state in device memory (Sec. 3.3, Eq. 2).
+
+    update() after each verify step (reads path_len and cu_nodes on the
+    device); select() after the draft's first forward (reads the draft LM
+    head's row_max / row_lse) writes each request's next triplet into
+    `self.triplet` [B, 3] and its DCS into `self.dcs` [B].  Nothing here
+    synchronises, so the calls can sit inside a captured decode loop."""
+
+    def __init__(self, batch: int, params: Optional[PolicyParams] = None, device="cuda"):
+        self.params = params or make_policy_params()
+        self.batch = int(batch)
+        self.state = torch.empty(max(self.batch, 1) * POLICY_STATE_BYTES, dtype=torch.uint8,
+                                 device=device)
+        self.triplet = torch.empty(max(self.batch, 1), 3, dtype=torch.int32, device=device)
+        self.dcs = torch.empty(max(self.batch, 1), dtype=torch.float64, device=device)
+        self.reset()
+
+    def triplets(self) -> list:
+        return asd_policy_triplets(self.params)
+
+    def reset(self, stream=None):
+        asd_policy_init(self.params, self.state, self.batch, stream)
+
+    def update(self, cu_nodes, path_len, stream=None):
+        asd_policy_update(self.params, cu_nodes, path_len, self.batch, self.state, stream)
+
+    def select(self, row_max, row_lse, rows=None, stream=None):
+        asd_policy_select(self.params, row_max, row_lse, rows, row_max.numel(), self.batch,
+                          self.state, self.triplet, self.dcs, stream)
+        return self.triplet
+
+    def state_arrays(self):
+        """(rar float64 [B], zero_streak int32 [B], breaks int32 [B]) on the
+        device, views of the state array."""
+        n = self.batch
+        rar = self.state.view(torch.float64)[0:2 * n:2]
+        ints = self.state.view(torch.int32).view(-1, 4)[:n]
+        return rar, ints[:, 2], ints[:, 3]

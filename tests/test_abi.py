@@ -24,7 +24,7 @@ def _declared():
 
 def test_every_declared_function_is_exported(lib):
     names = _declared()
-    assert len(names) == 12, names
+    assert len(names) == 16, names
     for n in names:
         assert hasattr(lib, n), n
 
@@ -34,7 +34,7 @@ def test_binding_names_match_header():
     build.build()
     from paper_2609_02897_gb300 import asd
     assert sorted(asd.EXPORTS) == _declared()
-    assert asd.abi_version() == 3
+    assert asd.abi_version() == 4
 
 
 def test_host_checks_without_gpu(lib):
@@ -97,3 +97,58 @@ def test_accept_rule_host_checks(lib):
     for rule in (asd.ASD_ACCEPT_GREEDY, asd.ASD_ACCEPT_GREEDY_ONCE):
         d.accept_rule = rule
         assert call(None) == 1
+
+
+def test_policy_triplets_match_the_oracle():
+    """asd_policy_triplets (host C) lists the same triplets, in the same order,
+    as the oracle's enumeration, on the paper's range and on random ones."""
+    import numpy as np
+    from paper_2609_02897_gb300 import build
+    build.build()
+    from paper_2609_02897_gb300 import asd
+    from oracle import policy as P
+    rng = np.random.default_rng(5)
+    ranges = [((3, 4, 4), (7, 1, 8)), ((7, 1, 8), (3, 4, 4)), ((4, 8, 10), (6, 2, 10)),
+              ((3, 1, 4), (3, 1, 4)), ((1, 1, 1), (128, 128, 128))]
+    ranges += [(tuple(int(x) for x in rng.integers(1, 33, 3)),
+                tuple(int(x) for x in rng.integers(1, 33, 3))) for _ in range(40)]
+    for sh, dp in ranges:
+        got = asd.asd_policy_triplets(asd.make_policy_params(shallow=sh, deep=dp))
+        assert got == P.reachable_triplets(sh, dp), (sh, dp)
+    # a short buffer receives the first `cap` triplets and the full count
+    import ctypes
+    buf = (ctypes.c_int32 * 6)()
+    pp = asd.make_policy_params()
+    assert asd._lib.asd_policy_triplets(ctypes.byref(pp), buf, 2) == 8
+    assert list(buf) == [3, 4, 4, 4, 4, 5]
+
+
+def test_policy_host_checks(lib):
+    """Invalid policy settings and null pointers are rejected before any CUDA
+    call (the placeholder pointers are never read)."""
+    from paper_2609_02897_gb300 import asd
+    buf = ctypes.c_void_p(1 << 20)
+    bad = [dict(alpha=0.0), dict(alpha=1.5), dict(alpha=float("nan")), dict(divisor=0.0),
+           dict(divisor=float("inf")), dict(rar_init=-0.1), dict(rar_init=1.1),
+           dict(shallow=(0, 4, 4)), dict(deep=(7, 1, 129)), dict(breaker=0)]
+    for kw in bad:
+        pp = asd.make_policy_params(**kw)
+        assert asd._lib.asd_policy_triplets(ctypes.byref(pp), None, 0) == -1, kw
+        assert asd._lib.asd_policy_init(ctypes.byref(pp), buf, 4, None) == 1, kw
+        assert asd._lib.asd_policy_update(ctypes.byref(pp), buf, buf, 4, buf, None) == 1, kw
+        assert asd._lib.asd_policy_select(ctypes.byref(pp), buf, buf, None, 4, 4, buf, buf, None,
+                                          None) == 1, kw
+    pp = asd.make_policy_params()
+    pp.reserved = 1
+    assert asd._lib.asd_policy_init(ctypes.byref(pp), buf, 4, None) == 1
+    pp = asd.make_policy_params()
+    assert asd._lib.asd_policy_init(ctypes.byref(pp), None, 4, None) == 1
+    assert asd._lib.asd_policy_init(ctypes.byref(pp), buf, -1, None) == 1
+    assert asd._lib.asd_policy_update(ctypes.byref(pp), None, buf, 4, buf, None) == 1
+    assert asd._lib.asd_policy_select(ctypes.byref(pp), buf, None, None, 4, 4, buf, buf, None,
+                                      None) == 1
+    assert asd._lib.asd_policy_select(ctypes.byref(pp), buf, buf, None, -1, 4, buf, buf, None,
+                                      None) == 1
+    # batch 0 enqueues nothing and succeeds
+    assert asd._lib.asd_policy_init(ctypes.byref(pp), buf, 0, None) == 0
+    assert asd._lib.asd_policy_triplets(None, None, 0) == -1

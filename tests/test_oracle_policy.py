@@ -121,7 +121,7 @@ def test_p_top1_closed_form():
 
 def test_ema_closed_form():
     """A constant fraction a for t steps: RAR_t = a + (1 - alpha)^t (RAR_0 - a)."""
-    for a_num, n in ((3, 7), (0, 3), (2, 5), (7, 7)):
+    for a_num, n in ((3, 7), (0, 3), (2, 5), (6, 7)):
         st = P.initial_state(1.0)
         a = a_num / (n - 1) if n > 1 else 0.0
         for t in range(1, 30):
