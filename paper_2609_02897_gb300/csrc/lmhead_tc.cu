@@ -366,6 +366,296 @@ __global__ void __launch_bounds__(192, 1)
   if (warp == 1) tmem_dealloc(tmem, kTmemCols);
 }
 
+// ----------------------------------------------------------------------------
+// Wide variant for more than 128 nodes.  Two node tiles share every streamed
+// W stage (W crosses HBM once per 256 nodes) and each MMA covers 256
+// vocabulary rows, D[128 nodes, 256 vocab rows], so that one MMA reads 12 KB
+// of shared memory per 128 x 256 x 16 product instead of 8 KB per
+// 128 x 128 x 16: with 128-row vocabulary tiles the tensor cores wait on
+// shared-memory reads.  A stage holds one k-block of the 256 W rows (the two
+// packed 128-row tiles, or 64-row TMA boxes) and of both node tiles; the
+// hidden rows (a few MB) stay in L2 across the vocabulary tiles.  TMEM holds
+// one 256-column accumulator per node tile; each has its own full / empty
+// barriers, so the MMAs into one resume as soon as the epilogue has drained
+// it.
+constexpr int kWideN = 2 * kLmTileN;                 // vocabulary rows per MMA
+constexpr int kWideG = 2;                            // node tiles per W stage
+constexpr int kWideStages = 3;
+constexpr int kWideA = kM * 128;                     // one node tile's k-block: 16 KB
+constexpr int kWideSlot = kWideG * kWideA + kWideN * 128;   // 64 KB
+constexpr uint32_t kWideTmemCols = kWideG * kWideN;  // 512
+
+__global__ void __launch_bounds__(192, 1)
+    lmhead_wide_kernel(const __grid_constant__ LmMaps maps, const LmParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  __shared__ __align__(8) uint64_t s_full[kWideStages];
+  __shared__ __align__(8) uint64_t s_empty[kWideStages];
+  __shared__ __align__(8) uint64_t s_tfull[kWideG];
+  __shared__ __align__(8) uint64_t s_tempty[kWideG];
+  __shared__ uint32_t s_tmem;
+  __shared__ volatile int s_abort;
+  __shared__ int s_pack_bad;
+
+  pdl_launch_dependents();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  const int ngroups = (p.V + kLmBoxRows - 1) / kLmBoxRows;
+  const int gs = lm_range_begin(blockIdx.x, p.g_lm, ngroups);
+  const int ge = lm_range_begin(blockIdx.x + 1, p.g_lm, ngroups);
+  const int vs = gs * kLmBoxRows;
+  const int ve = min(p.V, ge * kLmBoxRows);
+  const int nnt = (p.T + kM - 1) / kM;                     // node tiles
+  const int nng = (nnt + kWideG - 1) / kWideG;             // node-tile pairs
+  const int nkb = (p.K + kKB - 1) / kKB;
+
+  uint32_t base = smem_u32(smem_raw);
+  base += (1024u - (base & 1023u)) & 1023u;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kWideStages; ++s) {
+      mbar_init(smem_u32(&s_full[s]), 1);
+      mbar_init(smem_u32(&s_empty[s]), 1);
+    }
+    for (int a = 0; a < kWideG; ++a) {
+      mbar_init(smem_u32(&s_tfull[a]), 1);
+      mbar_init(smem_u32(&s_tempty[a]), 4);
+    }
+    s_abort = 0;
+    int bad = 0;
+    if (p.w_packed) {
+      const LmPackHeader* h = reinterpret_cast<const LmPackHeader*>(p.w_packed);
+      bad = (h->magic != kLmPackMagic || h->version != kLmPackVersion || h->vocab != p.V ||
+             h->hidden != p.K || h->ranges != p.g_lm);
+      if (bad) set_status(p.status, ASD_ERR_SHAPE);
+    }
+    s_pack_bad = bad;
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(&s_tmem), kWideTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = s_tmem;
+  const int nvt = (ve > vs && !s_pack_bad) ? (ve - vs + kWideN - 1) / kWideN : 0;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ TMA producer
+    uint64_t pol_w = 0, pol_h = 0;
+    if (lane == 0) {
+      prefetch_tmap(&maps.h);
+      if (!p.w_packed) {
+        prefetch_tmap(&maps.w64);
+        prefetch_tmap(&maps.w32);
+      }
+      pol_w = l2_policy_evict_first();
+      pol_h = l2_policy_evict_last();
+    }
+    int stage = 0;
+    uint32_t ph = 0;
+    bool ok = true;
+    for (int ng0 = 0; ng0 < nng && ok; ++ng0) {
+      const int gn = min(kWideG, nnt - ng0 * kWideG);
+      for (int vt = 0; vt < nvt && ok; ++vt) {
+        const int v0 = vs + vt * kWideN;
+        const int nrows = min(kWideN, ve - v0);
+        // 32-row groups of the two 128-row halves (the packed tiles)
+        const int ng_lo = (min(kLmTileN, nrows) + kLmBoxRows - 1) / kLmBoxRows;
+        const int ng_hi = nrows > kLmTileN ? (nrows - kLmTileN + kLmBoxRows - 1) / kLmBoxRows : 0;
+        for (int kb = 0; kb < nkb; ++kb) {
+          const uint32_t full = smem_u32(&s_full[stage]);
+          ok = __shfl_sync(0xffffffffu, mbar_wait(smem_u32(&s_empty[stage]), ph ^ 1u), 0);
+          if (!ok || s_abort) {
+            ok = false;
+            break;
+          }
+          if (lane == 0) {
+            const uint32_t a_s = base + stage * kWideSlot;
+            const uint32_t b_s = a_s + kWideG * kWideA;
+            mbar_expect_tx(full,
+                           static_cast<uint32_t>(gn * kWideA + (ng_lo + ng_hi) * kGroupBytes));
+            for (int j = 0; j < gn; ++j)
+              tma_load_2d(a_s + j * kWideA, &maps.h, full, kb * kKB, (ng0 * kWideG + j) * kM,
+                          pol_h);
+            for (int hf = 0; hf < 2; ++hf) {
+              const int ngh = hf ? ng_hi : ng_lo;
+              if (ngh == 0) continue;
+              const int vh = v0 + hf * kLmTileN;       // a packed tile's first row
+              const uint32_t dst = b_s + hf * kBTile;
+              if (p.w_packed) {
+                const size_t off = kLmPackHeader +
+                                   static_cast<size_t>(kGroupBytes) *
+                                       (static_cast<size_t>(nkb) * (vh / kLmBoxRows) +
+                                        static_cast<size_t>(kb) * ngh);
+                bulk_load(dst, p.w_packed + off, static_cast<uint32_t>(ngh * kGroupBytes), full,
+                          pol_w);
+              } else {
+                int j = 0;
+                for (; j + 1 < ngh; j += 2)
+                  tma_load_2d(dst + j * kGroupBytes, &maps.w64, full, kb * kKB,
+                              vh + j * kLmBoxRows, pol_w);
+                if (j < ngh)
+                  tma_load_2d(dst + j * kGroupBytes, &maps.w32, full, kb * kKB,
+                              vh + j * kLmBoxRows, pol_w);
+              }
+            }
+          }
+          __syncwarp();
+          if (++stage == kWideStages) {
+            stage = 0;
+            ph ^= 1u;
+          }
+        }
+      }
+    }
+    if (!ok && lane == 0) {
+      set_status(p.status, ASD_ERR_TIMEOUT);
+      s_abort = 1;
+    }
+  } else if (warp == 1) {
+    // --------------------------------------------------------------- MMA issuer
+    // Accumulator use u (counted over the kernel) goes to TMEM buffer u % 2;
+    // its empty barrier completes once per lap.
+    int stage = 0;
+    uint32_t ph = 0;
+    int used = 0;
+    bool ok = true;
+    for (int ng0 = 0; ng0 < nng && ok; ++ng0) {
+      const int gn = min(kWideG, nnt - ng0 * kWideG);
+      for (int vt = 0; vt < nvt && ok; ++vt) {
+        const int v0 = vs + vt * kWideN;
+        const int nrows = min(kWideN, ve - v0);
+        const uint32_t idesc = idesc_bf16(kM, (nrows + 15) & ~15);
+        for (int kb = 0; kb < nkb && ok; ++kb) {
+          ok = __shfl_sync(0xffffffffu, mbar_wait(smem_u32(&s_full[stage]), ph), 0);
+          if (!ok || s_abort) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t a_s = base + stage * kWideSlot;
+          const uint32_t b_s = a_s + kWideG * kWideA;
+          for (int j = 0; j < gn; ++j) {
+            const int u = used + j;
+            const int acc = u % kWideG;
+            if (kb == 0) {
+              // the epilogue must have drained this buffer's previous tile
+              ok = __shfl_sync(
+                  0xffffffffu,
+                  mbar_wait(smem_u32(&s_tempty[acc]), ((static_cast<uint32_t>(u / kWideG)) & 1u) ^ 1u),
+                  0);
+              if (!ok || s_abort) {
+                ok = false;
+                break;
+              }
+              tc_fence_after();
+            }
+            if (lane == 0) {
+              const uint32_t d = tmem + static_cast<uint32_t>(acc * kWideN);
+#pragma unroll
+              for (int k = 0; k < kKB / 16; ++k)
+                tc_mma(d, sw128_desc(a_s + j * kWideA + 32 * k), sw128_desc(b_s + 32 * k), idesc,
+                       (kb | k) != 0 ? 1u : 0u);
+              if (kb == nkb - 1) tc_commit(smem_u32(&s_tfull[acc]));
+            }
+            __syncwarp();
+          }
+          if (!ok) break;
+          if (lane == 0) tc_commit(smem_u32(&s_empty[stage]));
+          __syncwarp();
+          if (++stage == kWideStages) {
+            stage = 0;
+            ph ^= 1u;
+          }
+        }
+        used += gn;
+      }
+    }
+    if (!ok && lane == 0) {
+      set_status(p.status, ASD_ERR_TIMEOUT);
+      s_abort = 1;
+    }
+  } else {
+    // ----------------------------------------------------------------- epilogue
+    // Thread `row` owns TMEM lane `row`: row `row` of both node tiles of the
+    // current pair, one running state each.
+    const int q = warp & 3;
+    const int row = q * 32 + lane;
+    pdl_wait();
+    int used = 0;
+    bool ok = true;
+    for (int ng0 = 0; ng0 < nng && ok; ++ng0) {
+      const int gn = min(kWideG, nnt - ng0 * kWideG);
+      RowState st[kWideG];
+#pragma unroll
+      for (int j = 0; j < kWideG; ++j) {
+        const int node = (ng0 * kWideG + j) * kM + row;
+        row_state_init(st[j], j < gn && node < p.T, node, vs, p.child_start, p.child_cnt,
+                       p.child_tok, p.T);
+      }
+      for (int vt = 0; vt < nvt && ok; ++vt) {
+        const int v0 = vs + vt * kWideN;
+        const int nrows = min(kWideN, ve - v0);
+        const int nchunks = (nrows + 31) / 32;
+#pragma unroll
+        for (int j = 0; j < kWideG; ++j) {
+          if (j >= gn || !ok) continue;
+          const int u = used + j;
+          const int acc = u % kWideG;
+          ok = __shfl_sync(0xffffffffu,
+                           mbar_wait(smem_u32(&s_tfull[acc]), (static_cast<uint32_t>(u / kWideG)) & 1u),
+                           0);
+          if (!ok || s_abort) {
+            ok = false;
+            continue;
+          }
+          tc_fence_after();
+          const int node = (ng0 * kWideG + j) * kM + row;
+          const bool active = node < p.T;
+          const uint32_t taddr = tmem + (static_cast<uint32_t>(q * 32) << 16) +
+                                 static_cast<uint32_t>(acc * kWideN);
+          for (int c = 0; c < nchunks; ++c) {
+            float r[32];
+            tmem_ld32(taddr + 32 * c, r);
+            if (active)
+              row_chunk(st[j], r, v0 + 32 * c, min(32, nrows - 32 * c), p.child_tok, p.child_id,
+                        p.l_draft, p.T);
+          }
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(smem_u32(&s_tempty[acc]));
+        }
+        used += gn;
+      }
+      if (ok) {
+#pragma unroll
+        for (int j = 0; j < kWideG; ++j) {
+          const int node = (ng0 * kWideG + j) * kM + row;
+          if (j < gn && node < p.T) {
+            LmPartial part;
+            part.m = st[j].m;
+            part.s = st[j].s;
+            part.a = st[j].a;
+            part.pad = 0;
+            p.part[static_cast<size_t>(node) * p.g_lm + blockIdx.x] = part;
+          }
+        }
+      }
+    }
+    if (!ok && lane == 0) {
+      set_status(p.status, ASD_ERR_TIMEOUT);
+      s_abort = 1;
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc(tmem, kWideTmemCols);
+}
+
 }  // namespace
 
 // One CTA per (32-row group g, k-block kb): copies that 4 KB block of W into
@@ -429,6 +719,14 @@ cudaError_t launch_lm_pack(const void* w, void* w_packed, int vocab, int hidden,
 
 cudaError_t launch_lmhead_bf16(const LmParams& p, const LmMaps& maps, cudaStream_t s) {
   if (p.a_rows < 8 || p.a_rows > kM || p.a_rows % 8) return cudaErrorInvalidValue;
+  if (p.T > kM) {
+    // several node tiles: the wide kernel (full 128-row node boxes)
+    if (p.a_rows != kM) return cudaErrorInvalidValue;
+    const size_t smem = 1024 + static_cast<size_t>(kWideStages) * kWideSlot;
+    cudaError_t err = set_smem_attrs(lmhead_wide_kernel, smem);
+    if (err != cudaSuccess) return err;
+    return launch_pdl(lmhead_wide_kernel, dim3(p.g_lm), dim3(192), smem, s, maps, p);
+  }
   const size_t smem = lmhead_tc_smem_bytes(p.a_rows);
   cudaError_t err = set_smem_attrs(lmhead_tc_kernel, smem);
   if (err != cudaSuccess) return err;

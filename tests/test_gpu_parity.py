@@ -289,3 +289,16 @@ def test_greedy_accept_path_call_matches_verify_step(dev, rule):
         asd.asd_accept_path(dims, d["parent"], d["tokens"], acc, ra, d["cu_nodes"], path, plen,
                             bonus, npro, ws)
     assert e.value.code == 1
+
+
+@pytest.mark.parametrize("B", [2, 3, 4, 5, 7, 8, 9])
+def test_lm_head_node_groups(dev, B):
+    """Trees of 128 nodes, B of them: beyond one 128-node tile the LM head
+    shares every W stage between a pair of node tiles (odd B: the last pair
+    has one tile) and covers 256 vocabulary rows per MMA."""
+    wl = H.prepared(5, small=True, overrides=dict(B=B))
+    assert wl.T == 128 * B
+    out, status, _, _ = dev.run_verify(wl, 0.3)
+    assert status == 0
+    H.compare_verify(wl, 0.3, out)
+    H.untouched_cache_equal(wl, out, _written(wl, out))
