@@ -436,15 +436,19 @@ def run_asd(args):
     tpk, tpk_kind = tensor_peak()
     t_bytes, t_flops = sb / (peak * 1e9), fl / (tpk * 1e12)
     lm_flops = 2 * wl.T * wl.hidden_dim * wl.vocab
+    # up to one 128-node tile: the weight-streaming kernel; more: the wide one
+    lm_kernel = "lmhead_tc_kernel" if wl.T <= 128 else "lmhead_wide_kernel"
+    if wl.dtype != "bf16":
+        lm_kernel = "lmhead_f32_kernel"
     if lm_flops / lmb <= (tpk * 1e12) / (peak * 1e9):
-        lm_roofline = {"kernel": "lmhead_tc_kernel", "bound": "hbm", "achieved": achieved,
+        lm_roofline = {"kernel": lm_kernel, "bound": "hbm", "achieved": achieved,
                        "peak": peak, "unit": "GB/s", "frac": achieved / peak,
                        "peak_source": peak_kind + " hbm_gbs (MEASURED_PEAKS.json)",
                        "algorithmic_bytes_per_launch": lmb, "avg_launch_us": 1e3 * lm_ms,
                        "traffic": LMHEAD_TRAFFIC_BYTES if CONFIG == 2 and packed else None}
     else:
         tf = lm_flops / (lm_ms * 1e-3) / 1e12
-        lm_roofline = {"kernel": "lmhead_tc_kernel", "bound": "tensor", "achieved": tf,
+        lm_roofline = {"kernel": lm_kernel, "bound": "tensor", "achieved": tf,
                        "peak": tpk, "unit": "TFLOP/s", "frac": tf / tpk,
                        "peak_source": tpk_kind + " bf16_tflops (MEASURED_PEAKS.json)",
                        "algorithmic_flops_per_launch": lm_flops, "avg_launch_us": 1e3 * lm_ms,
