@@ -57,6 +57,9 @@ def parse():
                     help="margin threshold (default: the workload's first)")
     ap.add_argument("--lm-layout", default="packed", choices=["packed", "rows"],
                     help="LM-head weight as packed once at load (default) or as [V, K] rows")
+    ap.add_argument("--lm-schedule", default="every-row", choices=["every-row", "lazy"],
+                    help="LM-head rows: every node's (default) or, level by level, only those "
+                         "the accepted-path walk can reach")
     return ap.parse_args()
 
 
@@ -102,25 +105,39 @@ def esz(wl):
     return 2 if wl.dtype == "bf16" else 4
 
 
-def lmhead_bytes(wl):
-    """Algorithmic bytes of the LM-head kernel: W and the hidden states read once,
-    per-row statistics written."""
-    return (wl.vocab + wl.T) * wl.hidden_dim * esz(wl) + wl.T * 16
+def lmhead_bytes(wl, rows=None, passes=1):
+    """Algorithmic bytes of the LM head: W read once per pass, the hidden states of
+    the computed rows read once, per-row statistics written (every row and one pass
+    unless given)."""
+    rows = wl.T if rows is None else rows
+    return (passes * wl.vocab + rows) * wl.hidden_dim * esz(wl) + rows * 16
 
 
-def step_flops(wl):
+def lazy_work(wl, row_max):
+    """Rows the lazy schedule computed (row_max not NaN) and the tree levels they
+    span (one W pass each)."""
+    reach = ~np.isnan(row_max)
+    depth = np.zeros(wl.T, np.int64)
+    for b in range(wl.B):
+        s, e = int(wl.cu_nodes[b]), int(wl.cu_nodes[b + 1])
+        for i in range(s + 1, e):
+            depth[i] = depth[s + int(wl.parent[i])] + 1
+    return int(reach.sum()), int(depth[reach].max()) + 1 if reach.any() else 0
+
+
+def step_flops(wl, lm_rows=None):
     """Algorithmic flops of one verify step: 4*Hq*D per (query node, visible key)
-    in attention, 2*hidden*V per LM-head row."""
+    in attention, 2*hidden*V per computed LM-head row (every row unless given)."""
     import oracle
     keys = 0
     for b in range(wl.B):
         s, e = int(wl.cu_nodes[b]), int(wl.cu_nodes[b + 1])
         keys += (e - s) * int(wl.ctx_len[b])
         keys += sum(len(oracle.ancestors_of(wl.parent[s:e], i)) for i in range(e - s))
-    return 4 * keys * wl.Hq * wl.D + 2 * wl.T * wl.hidden_dim * wl.vocab
+    return 4 * keys * wl.Hq * wl.D + 2 * (wl.T if lm_rows is None else lm_rows) * wl.hidden_dim * wl.vocab
 
 
-def step_bytes(wl, mean_path):
+def step_bytes(wl, mean_path, lm_bytes=None):
     """Algorithmic bytes of one verify step (every input read once, outputs written)."""
     ctx = int(wl.ctx_len.sum())
     e = esz(wl)
@@ -128,7 +145,7 @@ def step_bytes(wl, mean_path):
             + wl.T * wl.Hkv * wl.D * 2 * e        # tree K and V
             + wl.T * wl.Hq * wl.D * 2 * e)        # Q read, O written
     commit = mean_path * wl.B * wl.Hkv * wl.D * 2 * 2 * e
-    return attn + lmhead_bytes(wl) + commit
+    return attn + (lmhead_bytes(wl) if lm_bytes is None else lm_bytes) + commit
 
 
 class Clocks:
@@ -331,6 +348,9 @@ def run_asd(args):
                          asd.ASD_BF16 if is_bf16 else asd.ASD_F32, wl.page_size,
                          wl.ctx_max, wl.num_pages, int(np.diff(wl.cu_nodes).max()), wl.max_path,
                          asd.ASD_LM_PACKED if packed else asd.ASD_LM_ROWS)
+    lazy = args.lm_schedule == "lazy"
+    if lazy:
+        dims.lm_head_schedule = asd.ASD_LM_LAZY_LEVELS
     w_lm = f(wl.w)
     if packed:
         # model load: the LM-head weight is repacked once into the streaming layout
@@ -429,17 +449,23 @@ def run_asd(args):
             dist.destroy_process_group()
         return
     peak, peak_kind = peaks()
-    lmb = lmhead_bytes(wl)
+    lm_rows, lm_passes = wl.T, 1
+    if lazy:
+        lm_rows, lm_passes = lazy_work(wl, step.out["row_max"].float().cpu().numpy())
+    lmb = lmhead_bytes(wl, lm_rows, lm_passes)
     achieved = lmb / (lm_ms * 1e-3) / 1e9
-    sb = step_bytes(wl, mean_path)
-    fl = step_flops(wl)
+    sb = step_bytes(wl, mean_path, lmb)
+    fl = step_flops(wl, lm_rows)
     tpk, tpk_kind = tensor_peak()
     t_bytes, t_flops = sb / (peak * 1e9), fl / (tpk * 1e12)
-    lm_flops = 2 * wl.T * wl.hidden_dim * wl.vocab
+    lm_flops = 2 * lm_rows * wl.hidden_dim * wl.vocab
     # up to one 128-node tile: the weight-streaming kernel; more: the wide one
     lm_kernel = "lmhead_tc_kernel" if wl.T <= 128 else "lmhead_wide_kernel"
     if wl.dtype != "bf16":
         lm_kernel = "lmhead_f32_kernel"
+    if lazy:
+        lm_kernel = (f"lmhead_wide_kernel + lazy_level_kernel, {lm_passes} non-empty levels of "
+                     f"{wl.max_path} (LM-head stage total)")
     if lm_flops / lmb <= (tpk * 1e12) / (peak * 1e9):
         lm_roofline = {"kernel": lm_kernel, "bound": "hbm", "achieved": achieved,
                        "peak": peak, "unit": "GB/s", "frac": achieved / peak,
@@ -462,6 +488,8 @@ def run_asd(args):
         "config": workload_config(wl),
         "lm_head_weight": ("packed once at load by asd_pack_lm_head (same bytes, streaming order)"
                            if packed else "[vocab, hidden] rows"),
+        "lm_head_schedule": (f"lazy levels: {lm_rows} of {wl.T} rows computed, {lm_passes} W passes"
+                             if lazy else "every row"),
         "hbm_gbs": sb / (ms * 1e-3) / 1e9, "hbm_frac_of_" + peak_kind: sb / (ms * 1e-3) / 1e9 / peak,
         # the whole step against the binding resource: the time its bytes take at
         # the measured copy bandwidth or its flops at the measured bf16 rate
@@ -475,7 +503,7 @@ def run_asd(args):
                       "step_with_stage_events": 1e3 * staged_ms,
                       "note": "second timed region with events between kernels (no overlap)"},
         "mean_path_len": mean_path,
-        "gpu_launches": K * N_STAGE_KERNELS,
+        "gpu_launches": K * (N_STAGE_KERNELS + (1 + 2 * wl.max_path - 1 if lazy else 0)),
         "clocks": clk,
         "e2e": e2e,
     }

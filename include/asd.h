@@ -53,7 +53,7 @@
 extern "C" {
 #endif
 
-#define ASD_ABI_VERSION 4
+#define ASD_ABI_VERSION 5
 #define ASD_MAX_TREE_NODES 128
 #define ASD_NUM_STAGE_EVENTS 5
 
@@ -96,6 +96,28 @@ typedef enum asd_lm_layout {
   ASD_LM_PACKED = 1  /* bf16 only: the buffer written by asd_pack_lm_head        */
 } asd_lm_layout;
 
+/* Which LM-head rows a call computes (asd_lmhead_margin, asd_verify_step).
+ *   ASD_LM_EVERY_ROW    every node's row (default).
+ *   ASD_LM_LAZY_LEVELS  only the rows the accepted-path walk can read: the
+ *       roots and the nodes whose every ancestor (root excluded) was
+ *       accepted, computed one tree level per pass over W (max_path passes,
+ *       the later ones empty when the accepted region ends).  A verdict needs
+ *       the parent's row (Eq. 1), so this is what a walk from the root can
+ *       reach; the committed path, bonus token, n_promoted and the cache are
+ *       those of ASD_LM_EVERY_ROW, and every computed row and verdict is
+ *       bit-identical to it.  Nodes not reached keep row_max = row_lse = NaN,
+ *       row_argmax = -1, ratio = l_draft = NaN and accept = 0.  Pays when the
+ *       levels cost fewer weight passes than the full tree costs in flops
+ *       (many sequences, few accepted nodes).  bf16 only; every tree must be
+ *       shallower than max_path (a reached node at depth max_path records
+ *       ASD_ERR_SHAPE).  The workspace grows by 2 x (T rounded up to 128) x
+ *       hidden x 2 bytes for the levels' hidden rows.  Not available in
+ *       asd_lmhead_margin_noalloc (ASD_ERR_SHAPE). */
+typedef enum asd_lm_schedule {
+  ASD_LM_EVERY_ROW = 0,
+  ASD_LM_LAZY_LEVELS = 1
+} asd_lm_schedule;
+
 /* Shapes of one verify step.  All fields are int32. */
 typedef struct asd_dims {
   int32_t batch;        /* B: number of sequences (trees)                      */
@@ -115,6 +137,7 @@ typedef struct asd_dims {
                            path (nodes, root included)                         */
   int32_t lm_head_layout; /* asd_lm_layout of w_lm                             */
   int32_t accept_rule;    /* asd_accept_rule of step 3                          */
+  int32_t lm_head_schedule; /* asd_lm_schedule                                  */
 } asd_dims;
 
 /* Bytes of device workspace that the calls below need for `total_nodes`

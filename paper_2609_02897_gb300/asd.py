@@ -22,6 +22,7 @@ _lib = ctypes.CDLL(_LIB_PATH)
 ASD_F32, ASD_BF16 = 0, 1
 ASD_LM_ROWS, ASD_LM_PACKED = 0, 1
 ASD_ACCEPT_LONGEST, ASD_ACCEPT_ONCE, ASD_ACCEPT_GREEDY, ASD_ACCEPT_GREEDY_ONCE = 0, 1, 2, 3
+ASD_LM_EVERY_ROW, ASD_LM_LAZY_LEVELS = 0, 1
 MAX_TREE_NODES = 128
 NUM_STAGE_EVENTS = 5
 STATUS = {0: "ASD_OK", 1: "ASD_ERR_INVALID_ARG", 2: "ASD_ERR_SHAPE", 3: "ASD_ERR_TREE",
@@ -45,7 +46,7 @@ class Dims(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int32) for n in (
         "batch", "num_q_heads", "num_kv_heads", "head_dim", "hidden", "vocab", "dtype",
         "page_size", "ctx_max", "num_pages", "max_nodes", "max_path", "lm_head_layout",
-        "accept_rule")]
+        "accept_rule", "lm_head_schedule")]
 
 
 _vp = ctypes.c_void_p
@@ -132,9 +133,11 @@ def abi_version() -> int:
 
 
 def make_dims(batch, num_q_heads, num_kv_heads, head_dim, hidden, vocab, dtype, page_size,
-              ctx_max, num_pages, max_nodes, max_path, lm_head_layout=0, accept_rule=0) -> Dims:
+              ctx_max, num_pages, max_nodes, max_path, lm_head_layout=0, accept_rule=0,
+              lm_head_schedule=0) -> Dims:
     return Dims(batch, num_q_heads, num_kv_heads, head_dim, hidden, vocab, dtype, page_size,
-                ctx_max, num_pages, max_nodes, max_path, lm_head_layout, accept_rule)
+                ctx_max, num_pages, max_nodes, max_path, lm_head_layout, accept_rule,
+                lm_head_schedule)
 
 
 def _ptr(t: Optional[torch.Tensor]):

@@ -89,6 +89,9 @@ bool dims_ok(const asd_dims* d) {
   if (d->lm_head_layout != ASD_LM_ROWS && d->lm_head_layout != ASD_LM_PACKED) return false;
   if (d->lm_head_layout == ASD_LM_PACKED && d->dtype != ASD_BF16) return false;
   if (d->accept_rule < ASD_ACCEPT_LONGEST || d->accept_rule > ASD_ACCEPT_GREEDY_ONCE) return false;
+  if (d->lm_head_schedule != ASD_LM_EVERY_ROW && d->lm_head_schedule != ASD_LM_LAZY_LEVELS)
+    return false;
+  if (d->lm_head_schedule == ASD_LM_LAZY_LEVELS && d->dtype != ASD_BF16) return false;
   return true;
 }
 
@@ -122,6 +125,12 @@ WsLayout layout(const asd_dims& d, int T, int nsm) {
   L.child_tok = off;   off = align256(off + 4 * static_cast<size_t>(T));
   L.child_id = off;    off = align256(off + 4 * static_cast<size_t>(T));
   L.lm_part = off;     off = align256(off + sizeof(LmPartial) * static_cast<size_t>(T) * L.g_lm);
+  if (d.lm_head_schedule == ASD_LM_LAZY_LEVELS) {
+    L.lz_cap = (T + 127) / 128 * 128;
+    L.lz_count = off;  off = align256(off + 4 * (static_cast<size_t>(d.max_path) + 1));
+    L.lz_rows = off;   off = align256(off + 4 * 2 * static_cast<size_t>(T));
+    L.lz_h = off;      off = align256(off + 2 * 2 * static_cast<size_t>(L.lz_cap) * d.hidden);
+  }
   L.total = off;
   return L;
 }
@@ -273,6 +282,90 @@ asd_status run_lmhead(const Ctx& c, const void* hidden, const void* w, float* l_
   return err == cudaSuccess ? ASD_OK : ASD_ERR_CUDA;
 }
 
+float ln_tau(float tau);
+
+// The lazy schedule (asd_lm_schedule): level 0 holds the roots; each level's
+// rows go through the wide LM head, then the level kernel merges them,
+// judges their children and lists the accepted ones for the next level.
+// Writes every output of the finalize stage for the rows it computes.
+asd_status run_lmhead_lazy(const Ctx& c, const void* hidden, const void* w,
+                           const int32_t* parent, const int32_t* tokens,
+                           const int32_t* cu_nodes, float tau, float* row_max,
+                           int32_t* row_argmax, float* row_lse, float* l_draft, float* ratio,
+                           uint8_t* accept) {
+  const asd_dims& d = c.d;
+  const int levels = d.max_path;
+  const size_t hbytes = 2 * static_cast<size_t>(c.L.lz_cap) * d.hidden;
+  void* h[2] = {ws_at<uint8_t>(c.ws, c.L.lz_h), ws_at<uint8_t>(c.ws, c.L.lz_h) + hbytes};
+  int32_t* rows[2] = {ws_at<int32_t>(c.ws, c.L.lz_rows), ws_at<int32_t>(c.ws, c.L.lz_rows) + c.T};
+  int* count = ws_at<int>(c.ws, c.L.lz_count);
+
+  LmParams p{};
+  p.w = w;
+  p.child_start = ws_at<int32_t>(c.ws, c.L.child_start);
+  p.child_cnt = ws_at<int32_t>(c.ws, c.L.child_cnt);
+  p.child_tok = ws_at<int32_t>(c.ws, c.L.child_tok);
+  p.child_id = ws_at<int32_t>(c.ws, c.L.child_id);
+  p.part = ws_at<LmPartial>(c.ws, c.L.lm_part);
+  p.l_draft = l_draft;
+  p.status = ws_at<int>(c.ws, c.L.status);
+  p.T = c.T;
+  p.K = d.hidden;
+  p.V = d.vocab;
+  p.g_lm = c.L.g_lm;
+  p.a_rows = 128;
+  LmMaps maps[2] = {};
+  for (int k = 0; k < 2; ++k) {
+    if (!make_tmap_bf16(&maps[k].h, h[k], d.hidden, c.L.lz_cap, 128)) return ASD_ERR_CUDA;
+    if (d.lm_head_layout == ASD_LM_ROWS &&
+        (!make_tmap_bf16(&maps[k].w64, w, d.hidden, d.vocab, 2 * kLmBoxRows) ||
+         !make_tmap_bf16(&maps[k].w32, w, d.hidden, d.vocab, kLmBoxRows)))
+      return ASD_ERR_CUDA;
+  }
+  if (d.lm_head_layout == ASD_LM_PACKED) p.w_packed = static_cast<const uint8_t*>(w);
+
+  LazyParams z{};
+  z.parent = parent;
+  z.tokens = tokens;
+  z.cu_nodes = cu_nodes;
+  z.seq_flags = ws_at<int>(c.ws, c.L.seq_flags);
+  z.child_start = p.child_start;
+  z.child_cnt = p.child_cnt;
+  z.child_id = p.child_id;
+  z.hidden = hidden;
+  z.part = p.part;
+  z.row_max = row_max;
+  z.row_argmax = row_argmax;
+  z.row_lse = row_lse;
+  z.l_draft = l_draft;
+  z.ratio = ratio;
+  z.accept = accept;
+  z.count = count;
+  z.status = p.status;
+  z.B = d.batch;
+  z.T = c.T;
+  z.K = d.hidden;
+  z.g_lm = c.L.g_lm;
+  z.last_level = levels - 1;
+  z.ln_tau = ln_tau(tau);
+  z.rows_next = rows[0];
+  z.h_next = h[0];
+  if (launch_lazy_init(z, levels, c.st) != cudaSuccess) return ASD_ERR_CUDA;
+  const int nsm = device_sm_count();
+  for (int lv = 0; lv < levels; ++lv) {
+    p.hidden = h[lv & 1];
+    p.t_dev = count + lv;
+    p.row_node = rows[lv & 1];
+    if (launch_lmhead_bf16(p, maps[lv & 1], c.st) != cudaSuccess) return ASD_ERR_CUDA;
+    z.level = lv;
+    z.rows_cur = rows[lv & 1];
+    z.rows_next = rows[(lv + 1) & 1];
+    z.h_next = h[(lv + 1) & 1];
+    if (launch_lazy_level(z, nsm, c.st) != cudaSuccess) return ASD_ERR_CUDA;
+  }
+  return ASD_OK;
+}
+
 TailParams tail_params(const Ctx& c, int mode) {
   TailParams t{};
   t.mode = mode;
@@ -394,6 +487,9 @@ asd_status asd_lmhead_margin(const asd_dims* dims, const void* hidden, const voi
   if (launch_tree_prep(prep_params(c, parent, tokens, cu_nodes, nullptr, l_draft), c.st) !=
       cudaSuccess)
     return ASD_ERR_CUDA;
+  if (c.d.lm_head_schedule == ASD_LM_LAZY_LEVELS)
+    return run_lmhead_lazy(c, hidden, w_lm, parent, tokens, cu_nodes, tau, row_max, row_argmax,
+                           row_lse, l_draft, ratio, accept);
   st = run_lmhead(c, hidden, w_lm, l_draft);
   if (st != ASD_OK) return st;
   TailParams t = tail_params(c, kTailFinalize);
@@ -491,15 +587,20 @@ asd_status asd_verify_step(const asd_dims* dims, const asd_verify_args* a, void*
   record(a->stage_events[1], c.st);
   // The LM head goes first and takes one CTA per SM; the attention kernel
   // starts right behind it (it reads no output of the LM head) and its CTAs
-  // share the SMs with the LM head's while the weights stream in.
-  st = run_lmhead(c, a->hidden, a->w_lm, a->l_draft);
+  // share the SMs with the LM head's while the weights stream in.  The lazy
+  // schedule also finalises the rows it computes, so the tail only walks.
+  const bool lazy = c.d.lm_head_schedule == ASD_LM_LAZY_LEVELS;
+  st = lazy ? run_lmhead_lazy(c, a->hidden, a->w_lm, a->parent, a->tokens, a->cu_nodes, a->tau,
+                              a->row_max, a->row_argmax, a->row_lse, a->l_draft, a->ratio,
+                              a->accept)
+            : run_lmhead(c, a->hidden, a->w_lm, a->l_draft);
   if (st != ASD_OK) return st;
   record(a->stage_events[2], c.st);
   st = run_attention(c, a->q, a->k_cache, a->v_cache, a->page_table, a->ctx_len, a->tree_k,
                      a->tree_v, a->parent, a->cu_nodes, a->attn_out);
   if (st != ASD_OK) return st;
   record(a->stage_events[3], c.st);
-  TailParams t = tail_params(c, kTailFinalize | kTailWalk | kTailCompact);
+  TailParams t = tail_params(c, (lazy ? 0 : kTailFinalize) | kTailWalk | kTailCompact);
   t.parent = a->parent;
   t.tokens = a->tokens;
   t.cu_nodes = a->cu_nodes;
@@ -600,6 +701,7 @@ extern "C" asd_status asd_lmhead_margin_noalloc(
   if (!aligned16(hidden) || !aligned16(w_lm)) return ASD_ERR_INVALID_ARG;
   if (!dims_ok(dims)) return dims ? ASD_ERR_SHAPE : ASD_ERR_INVALID_ARG;
   if (!nodes_ok(dims, total_nodes)) return ASD_ERR_SHAPE;
+  if (dims->lm_head_schedule != ASD_LM_EVERY_ROW) return ASD_ERR_SHAPE;
   const int nsm = device_sm_count();
   if (nsm <= 0) return ASD_ERR_CUDA;
   Ctx c;

@@ -43,12 +43,37 @@ struct WsLayout {
   int n_splits;        // context splits of the attention kernel
   int split_len;       // keys per context split (multiple of 64)
   int n_parts;         // = n_splits (the tree keys ride with the last split)
+  // lazy LM-head schedule only (0 otherwise)
+  size_t lz_count;     // int32[max_path + 1]: rows per level
+  size_t lz_rows;      // int32[2][T]: node ids of a level's rows (two levels in flight)
+  size_t lz_h;         // bf16[2][lz_cap][hidden]: their hidden rows
+  int lz_cap;          // T rounded up to 128
 };
 
 // ---------------------------------------------------------------- device utils
 
 __device__ __forceinline__ void set_status(int* status, int code) {
   atomicCAS(status, 0, code);
+}
+
+// Folds one vocabulary range's LM-head statistics (max m2, sum of exp(logit -
+// m2) s2, lowest argmax a2) into a running (m, s, a); ties in the max keep the
+// lowest vocabulary id.  The merge of every row's partials (tail kernel and
+// lazy level kernel) uses this, in the same order.
+__device__ __forceinline__ void merge_part(float& m, float& s, int& a, float m2, float s2,
+                                           int a2) {
+  if (m2 == -INFINITY) return;
+  if (m == -INFINITY) {
+    m = m2;
+    s = s2;
+    a = a2;
+    return;
+  }
+  const float M = fmaxf(m, m2);
+  s = s * exp2f((m - M) * kLog2e) + s2 * exp2f((m2 - M) * kLog2e);
+  if (m2 > m) a = a2;
+  else if (m2 == m) a = min(a, a2);
+  m = M;
 }
 
 // Programmatic dependent launch: a kernel launched with programmatic stream

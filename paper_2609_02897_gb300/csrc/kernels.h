@@ -101,6 +101,11 @@ struct LmParams {
   int a_rows;               // node rows per hidden-state TMA box: min(128, T rounded to 8);
                             // accumulator rows past it belong to no node
   const uint8_t* w_packed;  // W in the packed streaming layout, or null ([V, K] rows via TMA)
+  // Lazy LM head (one tree level per launch): the number of hidden rows is
+  // read from *t_dev (at most T), written by the previous kernel; row r
+  // belongs to node row_node[r].  Both null: T rows, row r = node r.
+  const int* t_dev;
+  const int32_t* row_node;
 };
 constexpr int kLmStages = 3;       // 3 x 48 KB (a_rows <= 64): room for an attention CTA
 constexpr int kLmTileN = 128;      // vocabulary rows per MMA tile
@@ -179,5 +184,34 @@ struct TailParams {
   int ctx_max, page_size, pages_per_seq, num_pages;
 };
 cudaError_t launch_tail(const TailParams& p, cudaStream_t s);
+
+// Lazy, level-synchronous LM head: rows are computed for the roots and for
+// nodes reached through accepted nodes only, one tree level per LM-head pass.
+struct LazyParams {
+  const int32_t* parent;
+  const int32_t* tokens;
+  const int32_t* cu_nodes;
+  const int* seq_flags;
+  const int32_t* child_start;
+  const int32_t* child_cnt;
+  const int32_t* child_id;
+  const void* hidden;         // [T, K] bf16
+  const LmPartial* part;      // [rows of the level][g_lm]
+  float* row_max;
+  int32_t* row_argmax;
+  float* row_lse;
+  const float* l_draft;
+  float* ratio;
+  uint8_t* accept;
+  int* count;                 // [levels + 1] rows per level
+  int32_t* rows_cur;          // node ids of this level's rows
+  int32_t* rows_next;
+  void* h_next;               // [cap, K] bf16: hidden rows of the next level
+  int* status;
+  int B, T, K, g_lm, level, last_level;
+  float ln_tau;
+};
+cudaError_t launch_lazy_init(const LazyParams& p, int levels, cudaStream_t s);
+cudaError_t launch_lazy_level(const LazyParams& p, int nsm, cudaStream_t s);
 
 }  // namespace asd

@@ -398,13 +398,20 @@ __global__ void __launch_bounds__(192, 1)
 
   pdl_launch_dependents();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  // hidden rows of this launch: T, or (one level of the lazy schedule) the
+  // count and the rows that the previous kernel wrote
+  int nrow = p.T;
+  if (p.t_dev) {
+    pdl_wait();
+    nrow = min(max(*p.t_dev, 0), p.T);
+  }
 
   const int ngroups = (p.V + kLmBoxRows - 1) / kLmBoxRows;
   const int gs = lm_range_begin(blockIdx.x, p.g_lm, ngroups);
   const int ge = lm_range_begin(blockIdx.x + 1, p.g_lm, ngroups);
   const int vs = gs * kLmBoxRows;
   const int ve = min(p.V, ge * kLmBoxRows);
-  const int nnt = (p.T + kM - 1) / kM;                     // node tiles
+  const int nnt = (nrow + kM - 1) / kM;                    // node tiles
   const int nng = (nnt + kWideG - 1) / kWideG;             // node-tile pairs
   const int nkb = (p.K + kKB - 1) / kKB;
 
@@ -589,11 +596,13 @@ __global__ void __launch_bounds__(192, 1)
     for (int ng0 = 0; ng0 < nng && ok; ++ng0) {
       const int gn = min(kWideG, nnt - ng0 * kWideG);
       RowState st[kWideG];
+      bool act[kWideG];
 #pragma unroll
       for (int j = 0; j < kWideG; ++j) {
-        const int node = (ng0 * kWideG + j) * kM + row;
-        row_state_init(st[j], j < gn && node < p.T, node, vs, p.child_start, p.child_cnt,
-                       p.child_tok, p.T);
+        const int r = (ng0 * kWideG + j) * kM + row;
+        const int node = (j < gn && r < nrow && p.row_node) ? p.row_node[r] : r;
+        act[j] = j < gn && r < nrow && node >= 0 && node < p.T;
+        row_state_init(st[j], act[j], node, vs, p.child_start, p.child_cnt, p.child_tok, p.T);
       }
       for (int vt = 0; vt < nvt && ok; ++vt) {
         const int v0 = vs + vt * kWideN;
@@ -612,8 +621,7 @@ __global__ void __launch_bounds__(192, 1)
             continue;
           }
           tc_fence_after();
-          const int node = (ng0 * kWideG + j) * kM + row;
-          const bool active = node < p.T;
+          const bool active = act[j];
           const uint32_t taddr = tmem + (static_cast<uint32_t>(q * 32) << 16) +
                                  static_cast<uint32_t>(acc * kWideN);
           for (int c = 0; c < nchunks; ++c) {
@@ -632,14 +640,14 @@ __global__ void __launch_bounds__(192, 1)
       if (ok) {
 #pragma unroll
         for (int j = 0; j < kWideG; ++j) {
-          const int node = (ng0 * kWideG + j) * kM + row;
-          if (j < gn && node < p.T) {
+          const int r = (ng0 * kWideG + j) * kM + row;   // partials by row
+          if (j < gn && r < nrow) {
             LmPartial part;
             part.m = st[j].m;
             part.s = st[j].s;
             part.a = st[j].a;
             part.pad = 0;
-            p.part[static_cast<size_t>(node) * p.g_lm + blockIdx.x] = part;
+            p.part[static_cast<size_t>(r) * p.g_lm + blockIdx.x] = part;
           }
         }
       }
@@ -719,8 +727,9 @@ cudaError_t launch_lm_pack(const void* w, void* w_packed, int vocab, int hidden,
 
 cudaError_t launch_lmhead_bf16(const LmParams& p, const LmMaps& maps, cudaStream_t s) {
   if (p.a_rows < 8 || p.a_rows > kM || p.a_rows % 8) return cudaErrorInvalidValue;
-  if (p.T > kM) {
-    // several node tiles: the wide kernel (full 128-row node boxes)
+  if (p.T > kM || p.t_dev) {
+    // several node tiles, or a row count known on the device only: the wide
+    // kernel (full 128-row node boxes)
     if (p.a_rows != kM) return cudaErrorInvalidValue;
     const size_t smem = 1024 + static_cast<size_t>(kWideStages) * kWideSlot;
     cudaError_t err = set_smem_attrs(lmhead_wide_kernel, smem);

@@ -28,22 +28,6 @@ namespace {
 constexpr int kTailThreads = 1024;     // 32 warps: one node's merge per warp
 constexpr int kMaxPartsPerLane = kMaxLmRanges / 32;
 
-__device__ __forceinline__ void merge_part(float& m, float& s, int& a, float m2, float s2,
-                                           int a2) {
-  if (m2 == -INFINITY) return;
-  if (m == -INFINITY) {
-    m = m2;
-    s = s2;
-    a = a2;
-    return;
-  }
-  const float M = fmaxf(m, m2);
-  s = s * exp2f((m - M) * kLog2e) + s2 * exp2f((m2 - M) * kLog2e);
-  if (m2 > m) a = a2;
-  else if (m2 == m) a = min(a, a2);
-  m = M;
-}
-
 __global__ void __launch_bounds__(kTailThreads) tail_kernel(const TailParams p) {
   __shared__ int s_par[kMaxNodes];
   __shared__ int s_tok[kMaxNodes];

@@ -35,10 +35,11 @@ def dims_of(wl, max_path=None, max_nodes=None):
         max_path or wl.max_path)
 
 
-def run_verify(wl, tau, dev=None, stream=None, rule=0):
+def run_verify(wl, tau, dev=None, stream=None, rule=0, schedule=0):
     dev = dev or to_device(wl)
     dims = dims_of(wl)
     dims.accept_rule = rule
+    dims.lm_head_schedule = schedule
     step = asd.VerifyStep(dims, wl.T, attn_dtype=dtype_of(wl))
     step.bind(tau=tau, **dev)
     step.run(stream)

@@ -34,7 +34,7 @@ def test_binding_names_match_header():
     build.build()
     from paper_2609_02897_gb300 import asd
     assert sorted(asd.EXPORTS) == _declared()
-    assert asd.abi_version() == 4
+    assert asd.abi_version() == 5
 
 
 def test_host_checks_without_gpu(lib):
@@ -152,3 +152,16 @@ def test_policy_host_checks(lib):
     # batch 0 enqueues nothing and succeeds
     assert asd._lib.asd_policy_init(ctypes.byref(pp), buf, 0, None) == 0
     assert asd._lib.asd_policy_triplets(None, None, 0) == -1
+
+
+def test_lm_schedule_host_checks(lib):
+    """An unknown LM-head schedule, or the lazy one with fp32, fails the dims
+    check (ASD_ERR_SHAPE) before any CUDA call."""
+    from paper_2609_02897_gb300 import asd
+    buf = ctypes.c_void_p(1 << 20)
+    fn = asd._lib.asd_lmhead_margin
+    for dtype, sched in ((asd.ASD_BF16, 2), (asd.ASD_BF16, -1), (asd.ASD_F32, asd.ASD_LM_LAZY_LEVELS)):
+        d = asd.make_dims(1, 4, 4, 64, 256, 4096, dtype, 0, 64, 0, 8, 5, 0, 0, sched)
+        assert fn(ctypes.byref(d), buf, buf, buf, buf, buf, 8, ctypes.c_float(0.5), *([buf] * 6),
+                  buf, 1 << 20, None) == 2
+        assert lib.asd_workspace_bytes(ctypes.byref(d), 8) == 0
