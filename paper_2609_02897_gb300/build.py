@@ -17,7 +17,7 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 OUT_DIR = os.path.join(HERE, "_lib")
 LIB_PATH = os.path.join(OUT_DIR, "libasd.so")
-UNITS = ["tree_prep", "attention", "lmhead_tc", "lmhead_f32", "tail", "asd_api", "policy", "lazy"]
+UNITS = ["tree_prep", "attention", "attention_tc", "lmhead_tc", "lmhead_f32", "tail", "asd_api", "policy", "lazy"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

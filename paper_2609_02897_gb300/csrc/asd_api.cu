@@ -45,6 +45,21 @@ bool make_tmap_bf16(CUtensorMap* tm, const void* base, uint64_t cols, uint64_t r
              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// Tree K/V [T, Hkv, D] bf16 as a 3D map {D, Hkv, T}: a box of 64 columns x 1
+// head x box_nodes nodes lands as box_nodes rows of 128 bytes (128-byte swizzle).
+bool make_tree_tmap_bf16(CUtensorMap* tm, const void* base, uint64_t d, uint64_t hkv,
+                         uint64_t t, uint32_t box_nodes) {
+  EncodeTiledFn enc = encode_fn();
+  if (!enc) return false;
+  const cuuint64_t dims[3] = {d, hkv, t};
+  const cuuint64_t strides[2] = {d * 2, hkv * d * 2};
+  const cuuint32_t box[3] = {64, 1, box_nodes};
+  const cuuint32_t estr[3] = {1, 1, 1};
+  return enc(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box,
+             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 }  // namespace
 
 int asd::lm_ranges(int vocab, int nsm) {
@@ -117,6 +132,13 @@ WsLayout layout(const asd_dims& d, int T, int nsm) {
   L.split_len = ((per + 63) / 64) * 64;
   L.n_splits = std::max(1, (d.ctx_max + L.split_len - 1) / L.split_len);
   L.n_parts = L.n_splits;
+  // more than one 128-node tile: the LM head (wide kernel) leaves no room on
+  // its SMs, attention runs after it on the tensor-core kernel, unsplit
+  L.attn_tc = (d.dtype == ASD_BF16 && T > kAttnTcRows) ? 1 : 0;
+  if (L.attn_tc) {
+    L.n_splits = L.n_parts = 1;
+    L.split_len = std::max(d.ctx_max, 1);
+  }
   size_t off = 0;
   L.status = off;      off = align256(off + 16);
   L.seq_flags = off;   off = align256(off + 4 * static_cast<size_t>(d.batch));
@@ -225,7 +247,25 @@ asd_status run_attention(const Ctx& c, const void* q, const void* k_cache, const
   a.max_nodes = d.max_nodes;
   a.scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(d.head_dim)));
   cudaError_t err;
-  if (d.dtype == ASD_BF16) {
+  if (c.L.attn_tc) {
+    CUtensorMap tk, tv, ttk, ttv;
+    uint64_t rows;
+    uint32_t box_rows;
+    if (d.page_size == 0) {
+      rows = static_cast<uint64_t>(d.batch) * d.num_kv_heads * static_cast<uint64_t>(d.ctx_max);
+      box_rows = static_cast<uint32_t>(kAttnTcKeys);
+    } else {
+      rows = static_cast<uint64_t>(d.num_pages) * d.num_kv_heads * d.page_size;
+      box_rows = static_cast<uint32_t>(std::min(d.page_size, kAttnTcKeys));
+    }
+    if (rows == 0) rows = 1;  // no context at all: the map is never used
+    if (!make_tmap_bf16(&tk, k_cache, d.head_dim, rows, box_rows) ||
+        !make_tmap_bf16(&tv, v_cache, d.head_dim, rows, box_rows) ||
+        !make_tree_tmap_bf16(&ttk, tree_k, d.head_dim, d.num_kv_heads, c.T, kAttnTcKeys) ||
+        !make_tree_tmap_bf16(&ttv, tree_v, d.head_dim, d.num_kv_heads, c.T, kAttnTcKeys))
+      return ASD_ERR_CUDA;
+    err = launch_attention_tc(a, tk, tv, ttk, ttv, c.st);
+  } else if (d.dtype == ASD_BF16) {
     CUtensorMap tk, tv;
     uint64_t rows;
     uint32_t box_rows;

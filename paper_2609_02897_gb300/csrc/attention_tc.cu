@@ -1,0 +1,580 @@
+// Tree attention (Sec. 2 "Verify": the target scores every drafted node in
+// one forward pass) on the 5th-generation tensor cores, for steps where the
+// attention kernel has the SMs to itself (more than 128 tree nodes: the LM
+// head then takes most of an SM's shared memory and runs first).  bf16 in,
+// fp32 accumulate.
+//
+// Work item (one CTA): 128 query rows of one (sequence, KV head) pair, the
+// whole context.  The rows of a pair are its N nodes times the G query heads
+// that share the KV head, node-major (row r -> node r / G, head g*G + r % G);
+// row r lives in TMEM lane r.  Keys come in tiles of 128 through a 3-stage
+// TMA ring (128-byte swizzle; paged caches one box per page; the tree K/V
+// through a 3D map over [T, Hkv, D]); the last tile of a pair holds its tree
+// keys, where a node sees only its ancestors (bitmasks derived here from the
+// parent array).
+//
+//   Q             staged once into TMEM by the softmax warps
+//   S = Q . K^T   tcgen05.mma, A (= Q) from TMEM, K K-major in shared memory
+//   P = exp2(S*c - m), per row by the thread that owns the row, written back
+//                 over the tile's S columns as bf16 pairs
+//   O += P . V    tcgen05.mma, A (= P) from TMEM, V MN-major straight from its
+//                 TMA tile, O in TMEM for the whole item
+//
+// Every MMA thus reads one operand from shared memory.  The softmax keeps a
+// per-row reference max m and rescales O only when the running max exceeds m
+// by more than 2^8 in the exp2 domain (P then stays below 2^8 and the result
+// equals that with the exact running max).  S/P is double-buffered: the MMAs
+// of tile t+1 run while the softmax works on tile t.
+//
+// TMEM (512 columns): O [0, D), Q [128, 128 + D/2), S/P [256, 384) and
+// [384, 512).  Shared memory: the K/V ring, 3 x 64 KB for D = 128.
+// Warp roles (320 threads): warp 0 TMA producer, warp 1 TMEM allocator and
+// MMA issuer, warps 2-9 softmax and epilogue, two per TMEM lane quarter, each
+// on one half of every tile's keys.
+#include "kernels.h"
+#include "tc.cuh"
+
+namespace asd {
+namespace {
+
+constexpr int kRows = kAttnTcRows;   // query rows per CTA = TMEM lanes
+constexpr int kKeys = kAttnTcKeys;   // keys per tile
+constexpr int kStages = 3;           // K/V ring
+constexpr int kThreads = 320;
+constexpr int kSoftmaxThreads = 256;   // eight warps: two per TMEM lane quarter
+constexpr float kRescaleLog2 = 8.f;
+constexpr uint32_t kTmemCols = 512;
+constexpr uint32_t kQCol = 128;
+constexpr uint32_t kSCol0 = 256;
+
+// Dynamic shared memory, 1024-byte aligned: K [stage][D/64][128 keys][128 B],
+// then V likewise.
+template <int D>
+struct TcGeom {
+  static constexpr int kNH = D / 64;
+  static constexpr int kTileBytes = kNH * kKeys * 128;   // one K or one V tile
+  static constexpr int kKOff = 0;
+  static constexpr int kVOff = kStages * kTileBytes;
+  static constexpr int kBytes = kVOff + kStages * kTileBytes;
+};
+
+__device__ __forceinline__ bool anc_bit(uint64_t lo, uint64_t hi, int j) {
+  return j < 64 ? ((lo >> j) & 1ull) : ((hi >> (j - 64)) & 1ull);
+}
+
+// Named barrier 1 of the eight softmax warps.
+__device__ __forceinline__ void softmax_sync() {
+  asm volatile("bar.sync 1, %0;" ::"n"(kSoftmaxThreads) : "memory");
+}
+
+// AND of `v` over the eight softmax warps (named barrier 1); uniform result.
+__device__ __forceinline__ bool softmax_all(bool v) {
+  uint32_t r;
+  asm volatile(
+      "{\n\t.reg .pred p, q;\n\t"
+      "setp.ne.u32 q, %1, 0;\n\t"
+      "barrier.cta.red.and.pred p, 1, %2, q;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(r)
+      : "r"(v ? 1u : 0u), "n"(kSoftmaxThreads)
+      : "memory");
+  return r != 0;
+}
+
+// OR of `v` over the eight softmax warps (named barrier 1); uniform result.
+__device__ __forceinline__ bool softmax_any(bool v) {
+  uint32_t r;
+  asm volatile(
+      "{\n\t.reg .pred p, q;\n\t"
+      "setp.ne.u32 q, %1, 0;\n\t"
+      "barrier.cta.red.or.pred p, 1, %2, q;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(r)
+      : "r"(v ? 1u : 0u), "n"(kSoftmaxThreads)
+      : "memory");
+  return r != 0;
+}
+
+// Every lane polls (bounded); the result is lane 0's, uniform over the warp.
+__device__ __forceinline__ bool wait_all(uint64_t* bar, uint32_t parity) {
+  return __shfl_sync(0xffffffffu, mbar_wait(smem_u32(bar), parity) ? 1 : 0, 0) != 0;
+}
+
+__device__ __forceinline__ bool aborted_warp(volatile int* s_abort) {
+  return __shfl_sync(0xffffffffu, *s_abort, 0) != 0;
+}
+
+struct Item {
+  int b, g, s0, n, r0, nrows, R;
+  int ctx, nctx, ntree, ntiles;
+};
+
+__device__ __forceinline__ bool make_item(const AttnParams& p, Item& it) {
+  const int rb = blockIdx.x, bg = blockIdx.y;
+  it.b = bg / p.Hkv;
+  it.g = bg - it.b * p.Hkv;
+  it.s0 = p.cu_nodes[it.b];
+  it.n = p.cu_nodes[it.b + 1] - it.s0;
+  it.R = it.n * p.G;
+  it.r0 = rb * kRows;
+  // sequence extents and context lengths are caller inputs (the tree
+  // preparation reports bad ones); every access below stays in bounds anyway
+  if (it.n <= 0 || it.n > kMaxNodes || it.s0 < 0 || it.s0 + it.n > p.T || it.r0 >= it.R)
+    return false;
+  it.nrows = min(kRows, it.R - it.r0);
+  it.ctx = min(max(p.ctx_len[it.b], 0), p.ctx_max);
+  it.nctx = (it.ctx + kKeys - 1) / kKeys;
+  it.ntree = (it.n + kKeys - 1) / kKeys;
+  it.ntiles = it.nctx + it.ntree;
+  return true;
+}
+
+__device__ __forceinline__ size_t grow_of(const AttnParams& p, const Item& it, int r) {
+  const int rr = it.r0 + r;
+  const int i = rr / p.G;
+  return static_cast<size_t>(it.s0 + i) * p.Hq + it.g * p.G + (rr - i * p.G);
+}
+
+// Issues the K and V tiles of tile t into one stage (producer lane only).
+template <int D>
+__device__ __forceinline__ void issue_tile(const AttnParams& p, const Item& it, int t,
+                                           uint32_t k_s, uint32_t v_s, uint32_t bar,
+                                           const CUtensorMap* tm_k, const CUtensorMap* tm_v,
+                                           const CUtensorMap* tm_tk, const CUtensorMap* tm_tv,
+                                           uint64_t pol) {
+  using G = TcGeom<D>;
+  if (t >= it.nctx) {
+    // tree keys: rows s0 + key0 .. of KV head g (rows past T read as zeros)
+    const int key0 = (t - it.nctx) * kKeys;
+    mbar_expect_tx(bar, 2 * G::kTileBytes);
+#pragma unroll
+    for (int h = 0; h < G::kNH; ++h) {
+      tma_load_3d(k_s + h * (kKeys * 128), tm_tk, bar, h * 64, it.g, it.s0 + key0, pol);
+      tma_load_3d(v_s + h * (kKeys * 128), tm_tv, bar, h * 64, it.g, it.s0 + key0, pol);
+    }
+    return;
+  }
+  const int key0 = t * kKeys;
+  if (p.page_size == 0) {
+    const int row = (it.b * p.Hkv + it.g) * p.ctx_max + key0;
+    mbar_expect_tx(bar, 2 * G::kTileBytes);
+#pragma unroll
+    for (int h = 0; h < G::kNH; ++h) {
+      tma_load_2d(k_s + h * (kKeys * 128), tm_k, bar, h * 64, row, pol);
+      tma_load_2d(v_s + h * (kKeys * 128), tm_v, bar, h * 64, row, pol);
+    }
+    return;
+  }
+  // paged: one box of min(page, 128) rows per page the tile touches
+  const int ps = p.page_size;
+  const int br = ps < kKeys ? ps : kKeys;
+  const int nbox = kKeys / br;
+  int rows[kKeys / 8];
+  int cnt = 0;
+  for (int j = 0; j < nbox; ++j) {
+    const int key = key0 + j * br;
+    rows[j] = -1;
+    if (key >= it.ctx) continue;
+    const int page = p.page_table[static_cast<size_t>(it.b) * p.pages_per_seq + key / ps];
+    if (page < 0 || page >= p.num_pages) {
+      set_status(p.status, ASD_ERR_CTX_RANGE);
+      continue;
+    }
+    rows[j] = (page * p.Hkv + it.g) * ps + (key % ps);
+    ++cnt;
+  }
+  mbar_expect_tx(bar, static_cast<uint32_t>(cnt * 2 * G::kNH * br * 128));
+  for (int j = 0; j < nbox; ++j) {
+    if (rows[j] < 0) continue;
+#pragma unroll
+    for (int h = 0; h < G::kNH; ++h) {
+      tma_load_2d(k_s + h * (kKeys * 128) + j * br * 128, tm_k, bar, h * 64, rows[j], pol);
+      tma_load_2d(v_s + h * (kKeys * 128) + j * br * 128, tm_v, bar, h * 64, rows[j], pol);
+    }
+  }
+}
+
+// Softmax warps (eight): warp w handles TMEM lane quarter w % 4 (its 32 query
+// rows, one thread per row) and half h = (w - 2) / 4 of every tile's 128 keys.
+// Per tile: read its 64 S columns, mask, exchange the row's partial max with
+// the warp that holds the other half, keep the reference max, and write P
+// (bf16 pairs) over the tile's S columns: half h's keys go to P columns
+// [32h, 32h + 32), which overlap S columns that both halves have read before
+// the exchange.  The row sum stays split between the two threads of a row
+// until the end.  Returns false (uniformly over the eight warps) when a
+// bounded wait gave up; otherwise inv = 1 / (row sum), with O complete in
+// TMEM.
+template <int D>
+__device__ __forceinline__ bool softmax_role(const AttnParams& p, const Item& it, uint32_t tmem,
+                                             uint8_t* gbase, const uint64_t (*s_anc)[2],
+                                             float (*s_mx)[2][kRows], float (*s_l)[kRows],
+                                             uint64_t* q_ready, uint64_t* s_full,
+                                             uint64_t* p_full, uint64_t* pv_done,
+                                             volatile int* s_abort, float& inv) {
+  using G = TcGeom<D>;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int hf = (warp - 2) >> 2;              // key half of every tile
+  const int row = (warp & 3) * 32 + lane;      // = TMEM lane
+  const int tid = threadIdx.x - 64;            // 0..255
+  const uint32_t lane_base = tmem + (static_cast<uint32_t>((warp & 3) * 32) << 16);
+
+  // this half of the row's query -> TMEM columns kQCol + [hf D/4, (hf+1) D/4),
+  // bf16 pairs; zeros past nrows
+  {
+    const bool mine = row < it.nrows;
+    const uint4* qg = reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(p.q) +
+                                                     (mine ? grow_of(p, it, row) : 0) * D +
+                                                     hf * (D / 2));
+#pragma unroll
+    for (int c = 0; c < D / 64; ++c) {
+      uint32_t r[16];
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const uint4 v = mine ? qg[c * 4 + k] : make_uint4(0u, 0u, 0u, 0u);
+        r[4 * k] = v.x;
+        r[4 * k + 1] = v.y;
+        r[4 * k + 2] = v.z;
+        r[4 * k + 3] = v.w;
+      }
+      tmem_st16(lane_base + kQCol + hf * (D / 4) + 16 * c, r);
+    }
+  }
+  tc_fence_before();
+  __syncwarp();
+  if (lane == 0) mbar_arrive(smem_u32(q_ready));
+
+  uint64_t alo = 0, ahi = 0;
+  if (row < it.nrows) {
+    const int node = (it.r0 + row) / p.G;
+    alo = s_anc[node][0];
+    ahi = s_anc[node][1];
+  }
+  const float c = p.scale_log2;
+  float m_ref = -INFINITY, l = 0.f;
+  bool ok = true, bad = false;
+  for (int t = 0; t < it.ntiles; ++t) {
+    const int b = t & 1;
+    const uint32_t sb = lane_base + kSCol0 + b * kKeys;
+    const bool tree = t >= it.nctx;
+    const int key0 = tree ? (t - it.nctx) * kKeys : t * kKeys;
+    const int valid = min(kKeys, (tree ? it.n : it.ctx) - key0);
+    float x[64];
+    float mt = -INFINITY;
+    const bool here = !bad && wait_all(&s_full[b], (t >> 1) & 1) && !aborted_warp(s_abort);
+    if (here) {
+      tc_fence_after();
+      tmem_ld64(sb + 64 * hf, x);
+      if (tree || valid < kKeys) {
+#pragma unroll
+        for (int k = 0; k < 64; ++k) {
+          const int key = 64 * hf + k;
+          bool v = key < valid;
+          if (tree) v = v && anc_bit(alo, ahi, key0 + key);
+          x[k] = v ? x[k] : -INFINITY;
+        }
+      }
+#pragma unroll
+      for (int k = 0; k < 64; ++k) mt = fmaxf(mt, x[k]);
+      s_mx[b][hf][row] = mt;
+    }
+    // every softmax warp decides together whether to go on (no warp may be
+    // left waiting at a barrier), and the partial maxima become visible
+    ok = softmax_all(here);
+    if (!ok) break;
+    // the row's max over both halves (raw scores; the scale is positive)
+    mt = fmaxf(mt, s_mx[b][hf ^ 1][row]) * c;
+    const float mn = fmaxf(m_ref, mt);
+    const bool had = m_ref != -INFINITY;
+    const bool need = had ? (mn > m_ref + kRescaleLog2) : (mn != -INFINITY);
+    if (__any_sync(0xffffffffu, need && had)) {
+      // O holds earlier tiles of this row: rescale this half of it once
+      // O += P V of tile t-1 is done
+      // (a wait that gives up marks the thread; all leave at the next tile)
+      if (!wait_all(&pv_done[(t - 1) & 1], ((t - 1) >> 1) & 1)) {
+        bad = true;
+      } else {
+        tc_fence_after();
+        const float alpha = (need && had) ? exp2f(m_ref - mn) : 1.f;
+#pragma unroll 1
+        for (int cc = 0; cc < D / 64; ++cc) {
+          float o[32];
+          const uint32_t oc = lane_base + hf * (D / 2) + 32 * cc;
+          tmem_ld32(oc, o);
+#pragma unroll
+          for (int i = 0; i < 32; ++i) o[i] *= alpha;
+          tmem_st32(oc, o);
+        }
+      }
+    }
+    if (need) {
+      l = had ? l * exp2f(m_ref - mn) : 0.f;
+      m_ref = mn;
+    }
+    const float mu = (m_ref == -INFINITY) ? 0.f : m_ref;
+    uint32_t pk[32];
+#pragma unroll
+    for (int k = 0; k < 64; k += 2) {
+      const float p0 = ex2_approx(fmaf(x[k], c, -mu)), p1 = ex2_approx(fmaf(x[k + 1], c, -mu));
+      l += p0 + p1;
+      __nv_bfloat162 h = __floats2bfloat162_rn(p0, p1);
+      pk[k / 2] = *reinterpret_cast<uint32_t*>(&h);
+    }
+    tmem_st32u(sb + 32 * hf, pk);
+    if (valid < kKeys) {
+      // ragged tile: V rows past the last valid key may hold anything; zero
+      // them so that 0 * V stays 0
+      uint8_t* vt = gbase + G::kVOff + (t % kStages) * G::kTileBytes;
+      constexpr int kChunksPerRow = G::kNH * 8;
+      for (int i = tid; i < (kKeys - valid) * kChunksPerRow; i += kSoftmaxThreads) {
+        const int r = valid + i / kChunksPerRow, rem = i % kChunksPerRow;
+        *reinterpret_cast<uint4*>(vt + (rem >> 3) * (kKeys * 128) + r * 128 + (rem & 7) * 16) =
+            make_uint4(0u, 0u, 0u, 0u);
+      }
+      fence_proxy_async();  // the zeroed rows are read by the tensor cores
+    }
+    tc_fence_before();
+    __syncwarp();
+    if (lane == 0) mbar_arrive(smem_u32(&p_full[b]));
+  }
+  if (ok) {
+    const int last = it.ntiles - 1;
+    ok = !bad && wait_all(&pv_done[last & 1], (last >> 1) & 1) && !aborted_warp(s_abort);
+    if (ok) tc_fence_after();
+  }
+  if (softmax_any(!ok)) {
+    if (tid == 0) {
+      set_status(p.status, ASD_ERR_TIMEOUT);
+      *s_abort = 1;
+    }
+    return false;
+  }
+  // the row sum over both halves
+  s_l[hf][row] = l;
+  softmax_sync();
+  l += s_l[hf ^ 1][row];
+  inv = l > 0.f ? 1.f / l : 0.f;
+  return true;
+}
+
+template <int D>
+__global__ void __launch_bounds__(kThreads, 1)
+    attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_v,
+                   const __grid_constant__ CUtensorMap tm_tk,
+                   const __grid_constant__ CUtensorMap tm_tv, const AttnParams p) {
+  using G = TcGeom<D>;
+  extern __shared__ uint8_t smem_raw[];
+  __shared__ __align__(8) uint64_t s_kv_full[kStages];
+  __shared__ __align__(8) uint64_t s_kv_empty[kStages];
+  __shared__ __align__(8) uint64_t s_s_full[2];    // S of a tile in TMEM (MMA -> softmax)
+  __shared__ __align__(8) uint64_t s_p_full[2];    // P of a tile in TMEM (softmax -> MMA)
+  __shared__ __align__(8) uint64_t s_pv_done[2];   // O += P V of a tile done (MMA -> softmax)
+  __shared__ __align__(8) uint64_t s_q_ready;
+  __shared__ __align__(8) uint64_t s_mma_done;
+  __shared__ uint32_t s_tmem;
+  __shared__ volatile int s_abort;
+  __shared__ int s_par[kMaxNodes];
+  __shared__ uint64_t s_anc[kMaxNodes][2];
+  __shared__ float s_mx[2][2][kRows];   // [tile parity][key half][row]: partial row max
+  __shared__ float s_l[2][kRows];       // [key half][row]: partial row sum
+
+  pdl_launch_dependents();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  Item it;
+  if (!make_item(p, it)) {  // no query rows here (uniform over the CTA)
+    pdl_wait();
+    return;
+  }
+
+  uint32_t base = smem_u32(smem_raw);
+  const uint32_t pad = (1024u - (base & 1023u)) & 1023u;
+  uint8_t* gbase = smem_raw + pad;
+  base += pad;
+  const uint32_t k_s0 = base + G::kKOff, v_s0 = base + G::kVOff;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(smem_u32(&s_kv_full[s]), 1);
+      mbar_init(smem_u32(&s_kv_empty[s]), 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(smem_u32(&s_s_full[b]), 1);
+      mbar_init(smem_u32(&s_p_full[b]), kSoftmaxThreads / 32);
+      mbar_init(smem_u32(&s_pv_done[b]), 1);
+    }
+    mbar_init(smem_u32(&s_q_ready), kSoftmaxThreads / 32);
+    mbar_init(smem_u32(&s_mma_done), 1);
+    s_abort = 0;
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(&s_tmem), kTmemCols);
+    tmem_relinquish();
+  }
+  // ancestor bitmasks (self included) of the sequence's nodes for the tree
+  // tile; a malformed parent ends the walk, so it is bounded
+  for (int i = threadIdx.x; i < it.n; i += kThreads) s_par[i] = p.parent[it.s0 + i];
+  __syncthreads();
+  for (int i = threadIdx.x; i < it.n; i += kThreads) {
+    uint64_t lo = 0, hi = 0;
+    int u = i;
+    while (true) {
+      if (u < 64) lo |= 1ull << u; else hi |= 1ull << (u - 64);
+      const int pu = s_par[u];
+      if (pu < 0 || pu >= u) break;
+      u = pu;
+    }
+    s_anc[i][0] = lo;
+    s_anc[i][1] = hi;
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = s_tmem;
+
+  bool ok = false;           // softmax warps: O complete in TMEM
+  float inv = 0.f;
+  if (warp == 0) {
+    // ------------------------------------------------------------ TMA producer
+    if (lane == 0) {
+      prefetch_tmap(&tm_k);
+      prefetch_tmap(&tm_v);
+      prefetch_tmap(&tm_tk);
+      prefetch_tmap(&tm_tv);
+      const uint64_t pol = l2_policy_evict_first();
+      int issued = 0;
+      for (int t = 0; t < it.ntiles; ++t) {
+        const int stage = t % kStages;
+        if (!mbar_wait(smem_u32(&s_kv_empty[stage]), ((t / kStages) & 1) ^ 1u)) {
+          set_status(p.status, ASD_ERR_TIMEOUT);
+          s_abort = 1;
+          break;
+        }
+        if (s_abort) break;
+        issue_tile<D>(p, it, t, k_s0 + stage * G::kTileBytes, v_s0 + stage * G::kTileBytes,
+                      smem_u32(&s_kv_full[stage]), &tm_k, &tm_v, &tm_tk, &tm_tv, pol);
+        ++issued;
+      }
+      // every copy issued has landed before the buffers are reused or left
+      for (int t = max(0, issued - kStages); t < issued; ++t)
+        mbar_wait(smem_u32(&s_kv_full[t % kStages]), (t / kStages) & 1);
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    // --------------------------------------------------------------- MMA issuer
+    if (lane == 0) {
+      const uint32_t idesc_s = idesc_bf16(kRows, kKeys);         // S = Q K^T
+      const uint32_t idesc_o = idesc_bf16(kRows, D, true);       // O += P V, V MN-major
+      bool mok = mbar_wait(smem_u32(&s_q_ready), 0);
+      if (mok) tc_fence_after();
+      for (int t = 0; mok && t <= it.ntiles; ++t) {
+        if (t < it.ntiles) {
+          const int stage = t % kStages, b = t & 1;
+          mok = mbar_wait(smem_u32(&s_kv_full[stage]), (t / kStages) & 1);
+          // the S/P buffer is free once O += P V of tile t-2 is done
+          if (mok && t >= 2) mok = mbar_wait(smem_u32(&s_pv_done[b]), ((t >> 1) - 1) & 1);
+          if (!mok || s_abort) break;
+          tc_fence_after();
+          const uint32_t kst = k_s0 + stage * G::kTileBytes;
+#pragma unroll
+          for (int ks = 0; ks < D / 16; ++ks) {
+            const int h = ks >> 2, kk = ks & 3;
+            tc_mma_ts(tmem + kSCol0 + b * kKeys, tmem + kQCol + ks * 8,
+                      sw128_desc(kst + h * (kKeys * 128) + 32 * kk), idesc_s, ks > 0 ? 1u : 0u);
+          }
+          tc_commit(smem_u32(&s_s_full[b]));
+        }
+        if (t >= 1) {
+          // O += P_j V_j for the previous tile j, after its softmax
+          const int j = t - 1, stage = j % kStages, b = j & 1;
+          mok = mbar_wait(smem_u32(&s_p_full[b]), (j >> 1) & 1);
+          if (!mok || s_abort) break;
+          tc_fence_after();
+          const uint32_t vst = v_s0 + stage * G::kTileBytes;
+#pragma unroll
+          for (int kk = 0; kk < kKeys / 16; ++kk)
+            tc_mma_ts(tmem, tmem + kSCol0 + b * kKeys + kk * 8,
+                      sw128_desc_mn(vst + kk * 2048, kKeys * 128, 1024), idesc_o,
+                      (j > 0 || kk > 0) ? 1u : 0u);
+          tc_commit(smem_u32(&s_pv_done[b]));
+          tc_commit(smem_u32(&s_kv_empty[stage]));
+        }
+      }
+      if (!mok) {
+        set_status(p.status, ASD_ERR_TIMEOUT);
+        s_abort = 1;
+      }
+      // every MMA issued above has finished before TMEM or the buffers are reused
+      tc_commit(smem_u32(&s_mma_done));
+      mbar_wait(smem_u32(&s_mma_done), 0);
+    }
+    __syncwarp();
+  } else {
+    ok = softmax_role<D>(p, it, tmem, gbase, s_anc, s_mx, s_l, &s_q_ready, s_s_full, s_p_full,
+                         s_pv_done, &s_abort, inv);
+  }
+
+  // ------------------------------------------------------------------ finish
+  tc_fence_before();
+  __syncthreads();   // the tile buffers and the tensor cores are idle from here on
+  tc_fence_after();
+  if (warp >= 2 && ok) {
+    // each thread writes its key half's share of the row: D/2 output columns
+    const int hf = (warp - 2) >> 2;
+    const int row = (warp & 3) * 32 + lane;   // TMEM lane = query row
+    const uint32_t lane_base = tmem + (static_cast<uint32_t>((warp & 3) * 32) << 16) +
+                               static_cast<uint32_t>(hf * (D / 2));
+    const bool mine = row < it.nrows;
+    __nv_bfloat16* out = static_cast<__nv_bfloat16*>(p.out) +
+                         (mine ? grow_of(p, it, row) : 0) * D + hf * (D / 2);
+#pragma unroll 1
+    for (int c = 0; c < D / 64; ++c) {
+      float o[32];
+      tmem_ld32(lane_base + 32 * c, o);   // every lane takes part in the warp-wide load
+      if (mine) {
+#pragma unroll
+        for (int k = 0; k < 32; k += 8) {
+          uint4 pk;
+          __nv_bfloat162 h0 = __floats2bfloat162_rn(o[k] * inv, o[k + 1] * inv);
+          __nv_bfloat162 h1 = __floats2bfloat162_rn(o[k + 2] * inv, o[k + 3] * inv);
+          __nv_bfloat162 h2 = __floats2bfloat162_rn(o[k + 4] * inv, o[k + 5] * inv);
+          __nv_bfloat162 h3 = __floats2bfloat162_rn(o[k + 6] * inv, o[k + 7] * inv);
+          pk.x = *reinterpret_cast<uint32_t*>(&h0);
+          pk.y = *reinterpret_cast<uint32_t*>(&h1);
+          pk.z = *reinterpret_cast<uint32_t*>(&h2);
+          pk.w = *reinterpret_cast<uint32_t*>(&h3);
+          *reinterpret_cast<uint4*>(out + 32 * c + k) = pk;
+        }
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc(tmem, kTmemCols);
+  pdl_wait();   // the next kernel's wait covers every earlier kernel
+}
+
+}  // namespace
+
+size_t attention_tc_smem_bytes(int head_dim) {
+  return 1024 + static_cast<size_t>(head_dim == 64 ? TcGeom<64>::kBytes : TcGeom<128>::kBytes);
+}
+
+cudaError_t launch_attention_tc(const AttnParams& p, const CUtensorMap& tm_k,
+                                const CUtensorMap& tm_v, const CUtensorMap& tm_tk,
+                                const CUtensorMap& tm_tv, cudaStream_t s) {
+  const dim3 grid((p.max_nodes * p.G + kRows - 1) / kRows, p.B * p.Hkv, 1);
+  const size_t smem = attention_tc_smem_bytes(p.D);
+  cudaError_t err;
+  if (p.D == 64) {
+    err = set_smem_attrs(attn_tc_kernel<64>, smem);
+    if (err != cudaSuccess) return err;
+    return launch_pdl(attn_tc_kernel<64>, grid, dim3(kThreads), smem, s, tm_k, tm_v, tm_tk, tm_tv, p);
+  }
+  if (p.D != 128) return cudaErrorInvalidValue;
+  err = set_smem_attrs(attn_tc_kernel<128>, smem);
+  if (err != cudaSuccess) return err;
+  return launch_pdl(attn_tc_kernel<128>, grid, dim3(kThreads), smem, s, tm_k, tm_v, tm_tk, tm_tv, p);
+}
+
+}  // namespace asd

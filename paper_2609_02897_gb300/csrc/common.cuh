@@ -48,6 +48,7 @@ struct WsLayout {
   size_t lz_rows;      // int32[2][T]: node ids of a level's rows (two levels in flight)
   size_t lz_h;         // bf16[2][lz_cap][hidden]: their hidden rows
   int lz_cap;          // T rounded up to 128
+  int attn_tc;         // 1: the tensor-core attention kernel (attention has the SMs to itself)
 };
 
 // ---------------------------------------------------------------- device utils
@@ -156,6 +157,16 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* tma
       "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
       ".L2::cache_hint [%0], [%1, {%3, %4}], [%2], %5;" ::"r"(dst),
       "l"(reinterpret_cast<uint64_t>(tmap)), "r"(bar), "r"(x), "r"(y), "l"(policy)
+      : "memory");
+}
+
+// 3D tiled TMA load (coordinates x innermost) into shared memory.
+__device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap* tmap, uint32_t bar,
+                                            int x, int y, int z, uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      ".L2::cache_hint [%0], [%1, {%3, %4, %5}], [%2], %6;" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(tmap)), "r"(bar), "r"(x), "r"(y), "r"(z), "l"(policy)
       : "memory");
 }
 

@@ -85,6 +85,18 @@ cudaError_t launch_attention_bf16(const AttnParams& p, const CUtensorMap& tm_k,
 cudaError_t launch_attention_f32(const AttnParams& p, cudaStream_t s);
 int attention_row_blocks(int max_nodes, int G);
 int attention_keys_per_tile();   // context keys per K/V tile = TMA box rows
+// bf16 path on the 5th-generation tensor cores, for steps where attention has
+// the SMs to itself (more than 128 tree nodes): one CTA per (128 query rows,
+// sequence x KV head), the whole context, no splits (p.n_parts == 1).  tm_k /
+// tm_v: 2D maps over the cache rows with boxes of 64 columns x
+// min(kAttnTcKeys, rows per page) rows; tm_tk / tm_tv: 3D maps over the tree
+// K/V [T, Hkv, D] with boxes of 64 columns x 1 head x kAttnTcKeys nodes.
+constexpr int kAttnTcRows = 128;   // query rows per CTA
+constexpr int kAttnTcKeys = 128;   // keys per tile
+size_t attention_tc_smem_bytes(int head_dim);
+cudaError_t launch_attention_tc(const AttnParams& p, const CUtensorMap& tm_k,
+                                const CUtensorMap& tm_v, const CUtensorMap& tm_tk,
+                                const CUtensorMap& tm_tv, cudaStream_t s);
 
 // -------------------------------------------------------------------- LM head
 struct LmParams {

@@ -37,7 +37,8 @@ def test_verify_step_small(dev, cfg, tau):
 
 
 @pytest.mark.parametrize("over", [dict(D=64), dict(page_size=32), dict(page_size=64),
-                                  dict(page_size=8)])
+                                  dict(page_size=8), dict(page_size=16, D=64),
+                                  dict(page_size=256)])
 def test_verify_variants(dev, over):
     cfg = 5 if "page_size" in over else 2
     wl = H.prepared(cfg, small=True, overrides=over)
