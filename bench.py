@@ -39,6 +39,9 @@ STAGES = ("prep", "lmhead", "attention", "tail")   # order of the stage events
 # ncu capture summarised in profiles/verify_step_llama8b_b1_ctx2048_tree60.md;
 # set to None whenever lmhead_tc.cu changes until it is captured again.
 LMHEAD_TRAFFIC_BYTES = 1054301744
+# DRAM bytes (read + write) of one LM-head launch from an ncu capture, per workload
+# (packed weight): 60 nodes (lmhead_tc_kernel) and 907 nodes (lmhead_wide_kernel, 4 W passes)
+LMHEAD_TRAFFIC_BY_CONFIG = {2: LMHEAD_TRAFFIC_BYTES, 3: 4194889096}
 
 
 def parse():
@@ -471,7 +474,7 @@ def run_asd(args):
                        "peak": peak, "unit": "GB/s", "frac": achieved / peak,
                        "peak_source": peak_kind + " hbm_gbs (MEASURED_PEAKS.json)",
                        "algorithmic_bytes_per_launch": lmb, "avg_launch_us": 1e3 * lm_ms,
-                       "traffic": LMHEAD_TRAFFIC_BYTES if CONFIG == 2 and packed else None}
+                       "traffic": LMHEAD_TRAFFIC_BY_CONFIG.get(CONFIG) if packed and not lazy else None}
     else:
         tf = lm_flops / (lm_ms * 1e-3) / 1e12
         lm_roofline = {"kernel": lm_kernel, "bound": "tensor", "achieved": tf,
