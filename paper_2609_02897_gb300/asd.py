@@ -263,21 +263,40 @@ class VerifyStep:
 
     OUT_FIELDS = ("attn_out", "row_max", "row_argmax", "row_lse", "l_draft", "ratio", "accept",
                   "path", "path_len", "bonus", "n_promoted", "ctx_len_out")
+    # the walk's results and the per-node verdicts lead the output arena, so
+    # that one copy (`results`) brings back what a decode loop reads per step
+    RESULT_FIELDS = ("path", "path_len", "bonus", "n_promoted", "ctx_len_out", "accept", "row_lse")
 
     def __init__(self, dims: Dims, total_nodes: int, device="cuda", attn_dtype=torch.bfloat16):
         self.dims = dims
         self.T = int(total_nodes)
-        T, B = self.T, dims.batch
-        f32 = dict(dtype=torch.float32, device=device)
-        i32 = dict(dtype=torch.int32, device=device)
-        self.out = dict(
-            attn_out=torch.empty(T, dims.num_q_heads, dims.head_dim, dtype=attn_dtype, device=device),
-            row_max=torch.empty(T, **f32), row_argmax=torch.empty(T, **i32),
-            row_lse=torch.empty(T, **f32), l_draft=torch.empty(T, **f32),
-            ratio=torch.empty(T, **f32), accept=torch.empty(T, dtype=torch.uint8, device=device),
-            path=torch.empty(B, dims.max_path, **i32), path_len=torch.empty(B, **i32),
-            bonus=torch.empty(B, **i32), n_promoted=torch.empty(B, **i32),
-            ctx_len_out=torch.empty(B, **i32))
+        T, B, i32, f32 = self.T, dims.batch, torch.int32, torch.float32
+        shapes = dict(path=((B, dims.max_path), i32), path_len=((B,), i32), bonus=((B,), i32),
+                      n_promoted=((B,), i32), ctx_len_out=((B,), i32),
+                      accept=((T,), torch.uint8), row_lse=((T,), f32), row_max=((T,), f32),
+                      row_argmax=((T,), i32), l_draft=((T,), f32), ratio=((T,), f32),
+                      attn_out=((T, dims.num_q_heads, dims.head_dim), attn_dtype))
+        order = self.RESULT_FIELDS + tuple(f for f in self.OUT_FIELDS if f not in self.RESULT_FIELDS)
+        offs, off = {}, 0
+        for f in order:
+            shape, dt = shapes[f]
+            n = 1
+            for x in shape:
+                n *= x
+            offs[f] = off
+            off = (off + n * torch.empty((), dtype=dt).element_size() + 255) // 256 * 256
+            if f == self.RESULT_FIELDS[-1]:
+                self._results_bytes = off
+        self.arena = torch.empty(off, dtype=torch.uint8, device=device)
+        self.out = {}
+        for f in order:
+            shape, dt = shapes[f]
+            n = 1
+            for x in shape:
+                n *= x
+            nb = n * torch.empty((), dtype=dt).element_size()
+            self.out[f] = self.arena[offs[f]:offs[f] + nb].view(dt).view(*shape)
+        self.results = self.arena[:self._results_bytes]
         self.workspace = alloc_workspace(dims, T, device)
         self.args = VerifyArgs()
         self._keep = []
@@ -306,6 +325,24 @@ class VerifyStep:
 
     def device_status(self, stream=None) -> int:
         return asd_get_device_status(self.workspace, stream)
+
+    def capture(self, copies_in=(), copies_out=()):
+        """A CUDA graph of one step: the (device, host) input copies in
+        `copies_in`, the verify step, then the (host, device) result copies in
+        `copies_out` (host tensors pinned).  It is recorded on a private stream;
+        `replay()` runs the whole step on the current stream with one launch
+        from the host, as a decode loop replays one graph per tree shape."""
+        g = torch.cuda.CUDAGraph()
+        side = torch.cuda.Stream()
+        side.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.graph(g, stream=side):
+            for dst, src in copies_in:
+                dst.copy_(src, non_blocking=True)
+            self.run(side)
+            for dst, src in copies_out:
+                dst.copy_(src, non_blocking=True)
+        torch.cuda.current_stream().wait_stream(side)
+        return g
 
 
 # ------------------------------------------------------------ tree-shape policy

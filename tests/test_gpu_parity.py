@@ -303,3 +303,30 @@ def test_lm_head_node_groups(dev, B):
     assert status == 0
     H.compare_verify(wl, 0.3, out)
     H.untouched_cache_equal(wl, out, _written(wl, out))
+
+
+def test_captured_step_with_host_copies(dev):
+    """VerifyStep.capture: input copies from pinned host memory, the verify
+    step and the result copies to pinned host memory, replayed as one graph,
+    give the eagerly launched step's results."""
+    import torch
+    from paper_2609_02897_gb300 import asd
+    wl = H.prepared(3, small=True)
+    ref, status, _, _ = dev.run_verify(wl, 0.5)
+    assert status == 0
+    d = dev.to_device(wl)
+    host = {k: d[k].cpu().pin_memory() for k in ("q", "tree_k", "tree_v", "hidden", "tokens",
+                                                  "parent", "cu_nodes", "ctx_len")}
+    for k in host:
+        d[k].zero_()                         # only the captured copies bring the inputs
+    step = asd.VerifyStep(dev.dims_of(wl), wl.T, attn_dtype=dev.dtype_of(wl))
+    step.bind(tau=0.5, **d)
+    outs = ("path", "path_len", "bonus", "row_lse", "accept")
+    host_out = {k: torch.empty_like(step.out[k], device="cpu").pin_memory() for k in outs}
+    g = step.capture([(d[k], v) for k, v in host.items()],
+                     [(v, step.out[k]) for k, v in host_out.items()])
+    g.replay()
+    torch.cuda.synchronize()
+    assert step.device_status() == 0
+    for k in outs:
+        np.testing.assert_array_equal(host_out[k].numpy(), ref[k], err_msg=k)
