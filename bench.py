@@ -39,9 +39,9 @@ STAGES = ("prep", "lmhead", "attention", "tail")   # order of the stage events
 # ncu capture summarised in profiles/verify_step_llama8b_b1_ctx2048_tree60.md;
 # set to None whenever lmhead_tc.cu changes until it is captured again.
 LMHEAD_TRAFFIC_BYTES = 1054301744
-# DRAM bytes (read + write) of one LM-head launch from an ncu capture, per workload
-# (packed weight): 60 nodes (lmhead_tc_kernel) and 907 nodes (lmhead_wide_kernel, 4 W passes)
-LMHEAD_TRAFFIC_BY_CONFIG = {2: LMHEAD_TRAFFIC_BYTES, 3: 4194889096}
+# DRAM bytes (read + write) of one LM-head launch from an ncu capture of the current
+# kernel, per workload (packed weight): 60 nodes (lmhead_tc_kernel)
+LMHEAD_TRAFFIC_BY_CONFIG = {2: LMHEAD_TRAFFIC_BYTES}
 
 
 def parse():

@@ -368,23 +368,91 @@ __global__ void __launch_bounds__(192, 1)
 
 // ----------------------------------------------------------------------------
 // Wide variant for more than 128 nodes.  Two node tiles share every streamed
-// W stage (W crosses HBM once per 256 nodes) and each MMA covers 256
-// vocabulary rows, D[128 nodes, 256 vocab rows], so that one MMA reads 12 KB
-// of shared memory per 128 x 256 x 16 product instead of 8 KB per
-// 128 x 128 x 16: with 128-row vocabulary tiles the tensor cores wait on
-// shared-memory reads.  A stage holds one k-block of the 256 W rows (the two
-// packed 128-row tiles, or 64-row TMA boxes) and of both node tiles; the
-// hidden rows (a few MB) stay in L2 across the vocabulary tiles.  TMEM holds
-// one 256-column accumulator per node tile; each has its own full / empty
-// barriers, so the MMAs into one resume as soon as the epilogue has drained
-// it.
+// W stage and each MMA covers 256 vocabulary rows, D[128 nodes, 256 vocab
+// rows], so that one MMA reads 12 KB of shared memory per 128 x 256 x 16
+// product instead of 8 KB per 128 x 128 x 16: with 128-row vocabulary tiles
+// the tensor cores wait on shared-memory reads.  A stage holds one k-block of
+// the 256 W rows (two packed 128-row tiles, or 64-row TMA boxes) and of the
+// CTA's two node tiles; the hidden rows (a few MB) stay in L2 across the
+// vocabulary tiles.  TMEM holds one 256-column accumulator per node tile, each
+// with its own full / empty barriers, so the MMAs into one resume as soon as
+// the epilogue has drained it.
+//
+// CL = 2: the CTAs come in clusters of two that own two adjacent vocabulary
+// ranges together and take alternate node pairs.  Each CTA copies one of the
+// two 128-row halves of every W stage and multicasts it to both, so every SM
+// pulls 48 KB per stage instead of 64 and W crosses HBM once per four node
+// tiles.  A stage is refilled only after both CTAs' MMAs have read it (each
+// CTA's commit arrives on both CTAs' empty barriers); both CTAs run the same
+// sequence of stages, a CTA without a node pair in the last round still
+// copying its half.  Every thread keeps one running state per vocabulary
+// range and writes one partial per range, so the statistics are those of
+// CTAs that own one range each, bit for bit.
 constexpr int kWideN = 2 * kLmTileN;                 // vocabulary rows per MMA
-constexpr int kWideG = 2;                            // node tiles per W stage
+constexpr int kWideG = 2;                            // node tiles per W stage and CTA
 constexpr int kWideStages = 3;
 constexpr int kWideA = kM * 128;                     // one node tile's k-block: 16 KB
 constexpr int kWideSlot = kWideG * kWideA + kWideN * 128;   // 64 KB
 constexpr uint32_t kWideTmemCols = kWideG * kWideN;  // 512
+constexpr int kTileGroups = kLmTileN / kLmBoxRows;   // 32-row groups per packed tile
 
+__device__ __forceinline__ uint32_t cta_rank_in_cluster() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+
+__device__ __forceinline__ void cluster_barrier() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;"
+               ::: "memory");
+}
+
+// Bulk copy global -> shared of every CTA in `mask` (same offset, each CTA's
+// barrier at `bar`'s offset receives the bytes).
+__device__ __forceinline__ void bulk_load_mc(uint32_t dst, const void* src, uint32_t bytes,
+                                             uint32_t bar, uint16_t mask, uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.multicast::cluster"
+      ".L2::cache_hint [%0], [%1], %2, [%3], %4, %5;" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(src)), "r"(bytes), "r"(bar), "h"(mask), "l"(policy)
+      : "memory");
+}
+
+__device__ __forceinline__ void tma_load_2d_mc(uint32_t dst, const CUtensorMap* tmap, uint32_t bar,
+                                               int x, int y, uint16_t mask, uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      ".multicast::cluster.L2::cache_hint [%0], [%1, {%3, %4}], [%2], %5, %6;" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(tmap)), "r"(bar), "r"(x), "r"(y), "h"(mask), "l"(policy)
+      : "memory");
+}
+
+// Arrive on `bar` of every CTA in `mask` once this thread's earlier tcgen05
+// operations are done.
+__device__ __forceinline__ void tc_commit_mc(uint32_t bar, uint16_t mask) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
+      " [%0], %1;" ::"r"(bar), "h"(mask)
+      : "memory");
+}
+
+// The CTA's (cluster's) vocabulary: CL adjacent ranges, each cut into packed
+// 128-row tiles from its start; tile j of the concatenation.
+struct WideVocab {
+  int gs0, ge0, nt0;         // first range: 32-row groups [gs0, ge0), packed tiles
+  int gs1, ge1, nt1;         // second range (CL = 2), else empty
+  int ntiles;                // packed tiles of all ranges
+  __device__ __forceinline__ void tile(int j, int V, int& q, int& g0, int& ng, int& v0,
+                                       int& rows) const {
+    q = j < nt0 ? 0 : 1;
+    g0 = q ? gs1 + (j - nt0) * kTileGroups : gs0 + j * kTileGroups;
+    ng = min(kTileGroups, (q ? ge1 : ge0) - g0);
+    v0 = g0 * kLmBoxRows;
+    rows = min(ng * kLmBoxRows, V - v0);
+  }
+};
+
+template <int CL>
 __global__ void __launch_bounds__(192, 1)
     lmhead_wide_kernel(const __grid_constant__ LmMaps maps, const LmParams p) {
   extern __shared__ uint8_t smem_raw[];
@@ -392,12 +460,15 @@ __global__ void __launch_bounds__(192, 1)
   __shared__ __align__(8) uint64_t s_empty[kWideStages];
   __shared__ __align__(8) uint64_t s_tfull[kWideG];
   __shared__ __align__(8) uint64_t s_tempty[kWideG];
+  __shared__ __align__(8) uint64_t s_mma_done;
   __shared__ uint32_t s_tmem;
   __shared__ volatile int s_abort;
   __shared__ int s_pack_bad;
 
   pdl_launch_dependents();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int rank = CL == 2 ? static_cast<int>(cta_rank_in_cluster()) : 0;
+  const uint16_t both = static_cast<uint16_t>((1u << CL) - 1u);
   // hidden rows of this launch: T, or (one level of the lazy schedule) the
   // count and the rows that the previous kernel wrote
   int nrow = p.T;
@@ -407,12 +478,18 @@ __global__ void __launch_bounds__(192, 1)
   }
 
   const int ngroups = (p.V + kLmBoxRows - 1) / kLmBoxRows;
-  const int gs = lm_range_begin(blockIdx.x, p.g_lm, ngroups);
-  const int ge = lm_range_begin(blockIdx.x + 1, p.g_lm, ngroups);
-  const int vs = gs * kLmBoxRows;
-  const int ve = min(p.V, ge * kLmBoxRows);
-  const int nnt = (nrow + kM - 1) / kM;                    // node tiles
-  const int nng = (nnt + kWideG - 1) / kWideG;             // node-tile pairs
+  const int cid = blockIdx.x / CL;                       // the ranges cid*CL .. cid*CL+CL-1
+  WideVocab voc;
+  voc.gs0 = lm_range_begin(cid * CL, p.g_lm, ngroups);
+  voc.ge0 = lm_range_begin(cid * CL + 1, p.g_lm, ngroups);
+  voc.gs1 = CL == 2 ? voc.ge0 : 0;
+  voc.ge1 = CL == 2 ? lm_range_begin(cid * CL + 2, p.g_lm, ngroups) : 0;
+  voc.nt0 = (voc.ge0 - voc.gs0 + kTileGroups - 1) / kTileGroups;
+  voc.nt1 = (voc.ge1 - voc.gs1 + kTileGroups - 1) / kTileGroups;
+  voc.ntiles = voc.nt0 + voc.nt1;
+  const int nnt = (nrow + kM - 1) / kM;                  // node tiles
+  const int nng = (nnt + kWideG - 1) / kWideG;           // node-tile pairs
+  const int nit = (nng + CL - 1) / CL;                   // rounds: pair i*CL + rank in round i
   const int nkb = (p.K + kKB - 1) / kKB;
 
   uint32_t base = smem_u32(smem_raw);
@@ -421,12 +498,13 @@ __global__ void __launch_bounds__(192, 1)
   if (threadIdx.x == 0) {
     for (int s = 0; s < kWideStages; ++s) {
       mbar_init(smem_u32(&s_full[s]), 1);
-      mbar_init(smem_u32(&s_empty[s]), 1);
+      mbar_init(smem_u32(&s_empty[s]), CL);      // every CTA of the cluster reads the stage
     }
     for (int a = 0; a < kWideG; ++a) {
       mbar_init(smem_u32(&s_tfull[a]), 1);
       mbar_init(smem_u32(&s_tempty[a]), 4);
     }
+    mbar_init(smem_u32(&s_mma_done), 1);
     s_abort = 0;
     int bad = 0;
     if (p.w_packed) {
@@ -444,9 +522,12 @@ __global__ void __launch_bounds__(192, 1)
   }
   tc_fence_before();
   __syncthreads();
+  if (CL == 2) cluster_barrier();   // the peer's barriers exist before any multicast
   tc_fence_after();
   const uint32_t tmem = s_tmem;
-  const int nvt = (ve > vs && !s_pack_bad) ? (ve - vs + kWideN - 1) / kWideN : 0;
+  // 256-row vocabulary tiles (pairs of packed tiles); none when a packed
+  // weight does not match (both CTAs of a cluster read the same header)
+  const int nvt = s_pack_bad ? 0 : (voc.ntiles + 1) / 2;
 
   if (warp == 0) {
     // ------------------------------------------------------------ TMA producer
@@ -463,14 +544,21 @@ __global__ void __launch_bounds__(192, 1)
     int stage = 0;
     uint32_t ph = 0;
     bool ok = true;
-    for (int ng0 = 0; ng0 < nng && ok; ++ng0) {
-      const int gn = min(kWideG, nnt - ng0 * kWideG);
+    for (int it = 0; it < nit && ok; ++it) {
+      const int pi = it * CL + rank;                       // this CTA's node pair
+      const int gn = pi < nng ? min(kWideG, nnt - pi * kWideG) : 0;
       for (int vt = 0; vt < nvt && ok; ++vt) {
-        const int v0 = vs + vt * kWideN;
-        const int nrows = min(kWideN, ve - v0);
-        // 32-row groups of the two 128-row halves (the packed tiles)
-        const int ng_lo = (min(kLmTileN, nrows) + kLmBoxRows - 1) / kLmBoxRows;
-        const int ng_hi = nrows > kLmTileN ? (nrows - kLmTileN + kLmBoxRows - 1) / kLmBoxRows : 0;
+        int q[2], g0[2], ng[2], v0[2], rows[2];
+        int wbytes = 0;
+#pragma unroll
+        for (int hf = 0; hf < 2; ++hf) {
+          ng[hf] = 0;
+          g0[hf] = 0;
+          if (2 * vt + hf < voc.ntiles) {
+            voc.tile(2 * vt + hf, p.V, q[hf], g0[hf], ng[hf], v0[hf], rows[hf]);
+            wbytes += ng[hf] * kGroupBytes;
+          }
+        }
         for (int kb = 0; kb < nkb; ++kb) {
           const uint32_t full = smem_u32(&s_full[stage]);
           ok = __shfl_sync(0xffffffffu, mbar_wait(smem_u32(&s_empty[stage]), ph ^ 1u), 0);
@@ -481,31 +569,45 @@ __global__ void __launch_bounds__(192, 1)
           if (lane == 0) {
             const uint32_t a_s = base + stage * kWideSlot;
             const uint32_t b_s = a_s + kWideG * kWideA;
-            mbar_expect_tx(full,
-                           static_cast<uint32_t>(gn * kWideA + (ng_lo + ng_hi) * kGroupBytes));
+            // every W byte of the stage lands here (half of it from the peer)
+            mbar_expect_tx(full, static_cast<uint32_t>(gn * kWideA + wbytes));
             for (int j = 0; j < gn; ++j)
-              tma_load_2d(a_s + j * kWideA, &maps.h, full, kb * kKB, (ng0 * kWideG + j) * kM,
+              tma_load_2d(a_s + j * kWideA, &maps.h, full, kb * kKB, (pi * kWideG + j) * kM,
                           pol_h);
+#pragma unroll
             for (int hf = 0; hf < 2; ++hf) {
-              const int ngh = hf ? ng_hi : ng_lo;
-              if (ngh == 0) continue;
-              const int vh = v0 + hf * kLmTileN;       // a packed tile's first row
+              if (ng[hf] == 0 || (CL == 2 && hf != rank)) continue;   // the peer's half
               const uint32_t dst = b_s + hf * kBTile;
               if (p.w_packed) {
                 const size_t off = kLmPackHeader +
                                    static_cast<size_t>(kGroupBytes) *
-                                       (static_cast<size_t>(nkb) * (vh / kLmBoxRows) +
-                                        static_cast<size_t>(kb) * ngh);
-                bulk_load(dst, p.w_packed + off, static_cast<uint32_t>(ngh * kGroupBytes), full,
-                          pol_w);
+                                       (static_cast<size_t>(nkb) * g0[hf] +
+                                        static_cast<size_t>(kb) * ng[hf]);
+                if (CL == 2)
+                  bulk_load_mc(dst, p.w_packed + off, static_cast<uint32_t>(ng[hf] * kGroupBytes),
+                               full, both, pol_w);
+                else
+                  bulk_load(dst, p.w_packed + off, static_cast<uint32_t>(ng[hf] * kGroupBytes),
+                            full, pol_w);
               } else {
+                const int vh = g0[hf] * kLmBoxRows;
                 int j = 0;
-                for (; j + 1 < ngh; j += 2)
-                  tma_load_2d(dst + j * kGroupBytes, &maps.w64, full, kb * kKB,
-                              vh + j * kLmBoxRows, pol_w);
-                if (j < ngh)
-                  tma_load_2d(dst + j * kGroupBytes, &maps.w32, full, kb * kKB,
-                              vh + j * kLmBoxRows, pol_w);
+                for (; j + 1 < ng[hf]; j += 2) {
+                  if (CL == 2)
+                    tma_load_2d_mc(dst + j * kGroupBytes, &maps.w64, full, kb * kKB,
+                                   vh + j * kLmBoxRows, both, pol_w);
+                  else
+                    tma_load_2d(dst + j * kGroupBytes, &maps.w64, full, kb * kKB,
+                                vh + j * kLmBoxRows, pol_w);
+                }
+                if (j < ng[hf]) {
+                  if (CL == 2)
+                    tma_load_2d_mc(dst + j * kGroupBytes, &maps.w32, full, kb * kKB,
+                                   vh + j * kLmBoxRows, both, pol_w);
+                  else
+                    tma_load_2d(dst + j * kGroupBytes, &maps.w32, full, kb * kKB,
+                                vh + j * kLmBoxRows, pol_w);
+                }
               }
             }
           }
@@ -529,12 +631,16 @@ __global__ void __launch_bounds__(192, 1)
     uint32_t ph = 0;
     int used = 0;
     bool ok = true;
-    for (int ng0 = 0; ng0 < nng && ok; ++ng0) {
-      const int gn = min(kWideG, nnt - ng0 * kWideG);
+    for (int it = 0; it < nit && ok; ++it) {
+      const int pi = it * CL + rank;
+      const int gn = pi < nng ? min(kWideG, nnt - pi * kWideG) : 0;
       for (int vt = 0; vt < nvt && ok; ++vt) {
-        const int v0 = vs + vt * kWideN;
-        const int nrows = min(kWideN, ve - v0);
-        const uint32_t idesc = idesc_bf16(kM, (nrows + 15) & ~15);
+        // N covers the low half's rows, or all 128 of them and the high half's
+        int q, g0, ng, v0, rows_lo, rows_hi = 0;
+        voc.tile(2 * vt, p.V, q, g0, ng, v0, rows_lo);
+        if (2 * vt + 1 < voc.ntiles) voc.tile(2 * vt + 1, p.V, q, g0, ng, v0, rows_hi);
+        const int ncols = rows_hi > 0 ? kLmTileN + rows_hi : rows_lo;
+        const uint32_t idesc = idesc_bf16(kM, (ncols + 15) & ~15);
         for (int kb = 0; kb < nkb && ok; ++kb) {
           ok = __shfl_sync(0xffffffffu, mbar_wait(smem_u32(&s_full[stage]), ph), 0);
           if (!ok || s_abort) {
@@ -570,7 +676,13 @@ __global__ void __launch_bounds__(192, 1)
             __syncwarp();
           }
           if (!ok) break;
-          if (lane == 0) tc_commit(smem_u32(&s_empty[stage]));
+          // the stage is free for refilling once every CTA of the cluster has read it
+          if (lane == 0) {
+            if (CL == 2)
+              tc_commit_mc(smem_u32(&s_empty[stage]), both);
+            else
+              tc_commit(smem_u32(&s_empty[stage]));
+          }
           __syncwarp();
           if (++stage == kWideStages) {
             stage = 0;
@@ -584,30 +696,38 @@ __global__ void __launch_bounds__(192, 1)
       set_status(p.status, ASD_ERR_TIMEOUT);
       s_abort = 1;
     }
+    // every tcgen05 operation of this thread, the commits included, is done
+    // before the CTA leaves the cluster
+    if (lane == 0) {
+      tc_commit(smem_u32(&s_mma_done));
+      mbar_wait(smem_u32(&s_mma_done), 0);
+    }
+    __syncwarp();
   } else {
     // ----------------------------------------------------------------- epilogue
     // Thread `row` owns TMEM lane `row`: row `row` of both node tiles of the
-    // current pair, one running state each.
-    const int q = warp & 3;
-    const int row = q * 32 + lane;
+    // current pair, one running state per node tile and vocabulary range.
+    const int q4 = warp & 3;
+    const int row = q4 * 32 + lane;
     pdl_wait();
     int used = 0;
     bool ok = true;
-    for (int ng0 = 0; ng0 < nng && ok; ++ng0) {
-      const int gn = min(kWideG, nnt - ng0 * kWideG);
-      RowState st[kWideG];
+    for (int it = 0; it < nit && ok; ++it) {
+      const int pi = it * CL + rank;
+      const int gn = pi < nng ? min(kWideG, nnt - pi * kWideG) : 0;
+      RowState st[CL][kWideG];
       bool act[kWideG];
 #pragma unroll
       for (int j = 0; j < kWideG; ++j) {
-        const int r = (ng0 * kWideG + j) * kM + row;
+        const int r = (pi * kWideG + j) * kM + row;
         const int node = (j < gn && r < nrow && p.row_node) ? p.row_node[r] : r;
         act[j] = j < gn && r < nrow && node >= 0 && node < p.T;
-        row_state_init(st[j], act[j], node, vs, p.child_start, p.child_cnt, p.child_tok, p.T);
+#pragma unroll
+        for (int qq = 0; qq < CL; ++qq)
+          row_state_init(st[qq][j], act[j], node, (qq ? voc.gs1 : voc.gs0) * kLmBoxRows,
+                         p.child_start, p.child_cnt, p.child_tok, p.T);
       }
       for (int vt = 0; vt < nvt && ok; ++vt) {
-        const int v0 = vs + vt * kWideN;
-        const int nrows = min(kWideN, ve - v0);
-        const int nchunks = (nrows + 31) / 32;
 #pragma unroll
         for (int j = 0; j < kWideG; ++j) {
           if (j >= gn || !ok) continue;
@@ -621,15 +741,26 @@ __global__ void __launch_bounds__(192, 1)
             continue;
           }
           tc_fence_after();
-          const bool active = act[j];
-          const uint32_t taddr = tmem + (static_cast<uint32_t>(q * 32) << 16) +
+          const uint32_t taddr = tmem + (static_cast<uint32_t>(q4 * 32) << 16) +
                                  static_cast<uint32_t>(acc * kWideN);
-          for (int c = 0; c < nchunks; ++c) {
-            float r[32];
-            tmem_ld32(taddr + 32 * c, r);
-            if (active)
-              row_chunk(st[j], r, v0 + 32 * c, min(32, nrows - 32 * c), p.child_tok, p.child_id,
-                        p.l_draft, p.T);
+          // the two packed tiles of the 256 columns, each from its own vocabulary base
+#pragma unroll
+          for (int hf = 0; hf < 2; ++hf) {
+            if (2 * vt + hf >= voc.ntiles) break;
+            int q, g0, ng, v0, rows;
+            voc.tile(2 * vt + hf, p.V, q, g0, ng, v0, rows);
+            for (int c = 0; c < (rows + 31) / 32; ++c) {
+              float r[32];
+              tmem_ld32(taddr + hf * kLmTileN + 32 * c, r);
+              if (act[j]) {
+                if (CL == 2 && q == 1)
+                  row_chunk(st[CL - 1][j], r, v0 + 32 * c, min(32, rows - 32 * c), p.child_tok,
+                            p.child_id, p.l_draft, p.T);
+                else
+                  row_chunk(st[0][j], r, v0 + 32 * c, min(32, rows - 32 * c), p.child_tok,
+                            p.child_id, p.l_draft, p.T);
+              }
+            }
           }
           tc_fence_before();
           __syncwarp();
@@ -640,14 +771,17 @@ __global__ void __launch_bounds__(192, 1)
       if (ok) {
 #pragma unroll
         for (int j = 0; j < kWideG; ++j) {
-          const int r = (ng0 * kWideG + j) * kM + row;   // partials by row
+          const int r = (pi * kWideG + j) * kM + row;   // partials by row, one per range
           if (j < gn && r < nrow) {
-            LmPartial part;
-            part.m = st[j].m;
-            part.s = st[j].s;
-            part.a = st[j].a;
-            part.pad = 0;
-            p.part[static_cast<size_t>(r) * p.g_lm + blockIdx.x] = part;
+#pragma unroll
+            for (int qq = 0; qq < CL; ++qq) {
+              LmPartial part;
+              part.m = st[qq][j].m;
+              part.s = st[qq][j].s;
+              part.a = st[qq][j].a;
+              part.pad = 0;
+              p.part[static_cast<size_t>(r) * p.g_lm + cid * CL + qq] = part;
+            }
           }
         }
       }
@@ -662,6 +796,7 @@ __global__ void __launch_bounds__(192, 1)
   __syncthreads();
   tc_fence_after();
   if (warp == 1) tmem_dealloc(tmem, kWideTmemCols);
+  if (CL == 2) cluster_barrier();   // no multicast or remote arrive targets a CTA that left
 }
 
 }  // namespace
@@ -725,16 +860,42 @@ cudaError_t launch_lm_pack(const void* w, void* w_packed, int vocab, int hidden,
   return cudaGetLastError();
 }
 
+namespace {
+template <int CL>
+cudaError_t launch_wide(const LmParams& p, const LmMaps& maps, cudaStream_t s) {
+  const size_t smem = 1024 + static_cast<size_t>(kWideStages) * kWideSlot;
+  cudaError_t err = set_smem_attrs(lmhead_wide_kernel<CL>, smem);
+  if (err != cudaSuccess) return err;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(p.g_lm);
+  cfg.blockDim = dim3(192);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = CL;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 2;
+  return cudaLaunchKernelEx(&cfg, lmhead_wide_kernel<CL>, maps, p);
+}
+}  // namespace
+
 cudaError_t launch_lmhead_bf16(const LmParams& p, const LmMaps& maps, cudaStream_t s) {
   if (p.a_rows < 8 || p.a_rows > kM || p.a_rows % 8) return cudaErrorInvalidValue;
   if (p.T > kM || p.t_dev) {
     // several node tiles, or a row count known on the device only: the wide
-    // kernel (full 128-row node boxes)
+    // kernel (full 128-row node boxes).  Clusters of two pay when every CTA has
+    // at least two rounds of node pairs (the CTAs of a cluster move in lock
+    // step; with one round the coupling costs more than the halved W traffic
+    // saves), and when the ranges pair up
     if (p.a_rows != kM) return cudaErrorInvalidValue;
-    const size_t smem = 1024 + static_cast<size_t>(kWideStages) * kWideSlot;
-    cudaError_t err = set_smem_attrs(lmhead_wide_kernel, smem);
-    if (err != cudaSuccess) return err;
-    return launch_pdl(lmhead_wide_kernel, dim3(p.g_lm), dim3(192), smem, s, maps, p);
+    const int pairs = (p.T + kWideG * kM - 1) / (kWideG * kM);
+    const bool cluster = p.g_lm % 2 == 0 && !p.t_dev && pairs >= 4;
+    return cluster ? launch_wide<2>(p, maps, s) : launch_wide<1>(p, maps, s);
   }
   const size_t smem = lmhead_tc_smem_bytes(p.a_rows);
   cudaError_t err = set_smem_attrs(lmhead_tc_kernel, smem);
