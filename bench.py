@@ -40,8 +40,9 @@ STAGES = ("prep", "lmhead", "attention", "tail")   # order of the stage events
 # set to None whenever lmhead_tc.cu changes until it is captured again.
 LMHEAD_TRAFFIC_BYTES = 1054301744
 # DRAM bytes (read + write) of one LM-head launch from an ncu capture of the current
-# kernel, per workload (packed weight): 60 nodes (lmhead_tc_kernel)
-LMHEAD_TRAFFIC_BY_CONFIG = {2: LMHEAD_TRAFFIC_BYTES}
+# kernel, per workload (packed weight): 60 nodes (lmhead_tc_kernel) and 907 nodes
+# (lmhead_wide_kernel in clusters of two: 2 W passes)
+LMHEAD_TRAFFIC_BY_CONFIG = {2: LMHEAD_TRAFFIC_BYTES, 3: 2099486768}
 
 
 def parse():
