@@ -129,15 +129,22 @@ def lazy_work(wl, row_max):
     return int(reach.sum()), int(depth[reach].max()) + 1 if reach.any() else 0
 
 
+def tree_keys(parent):
+    """Tree keys a node sees: its ancestors and itself (node depth + 1)."""
+    depth = [0] * len(parent)
+    for i in range(1, len(parent)):
+        depth[i] = depth[int(parent[i])] + 1
+    return sum(depth) + len(parent)
+
+
 def step_flops(wl, lm_rows=None):
     """Algorithmic flops of one verify step: 4*Hq*D per (query node, visible key)
     in attention, 2*hidden*V per computed LM-head row (every row unless given)."""
-    import oracle
     keys = 0
     for b in range(wl.B):
         s, e = int(wl.cu_nodes[b]), int(wl.cu_nodes[b + 1])
         keys += (e - s) * int(wl.ctx_len[b])
-        keys += sum(len(oracle.ancestors_of(wl.parent[s:e], i)) for i in range(e - s))
+        keys += tree_keys(wl.parent[s:e])
     return 4 * keys * wl.Hq * wl.D + 2 * (wl.T if lm_rows is None else lm_rows) * wl.hidden_dim * wl.vocab
 
 
