@@ -526,8 +526,11 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const __grid_constant__ 
 }
 
 // ----------------------------------------------------------- fp32 SIMT path
-// One warp per query row; lanes split the head dimension.  Exact fp32 math for
-// the fp32 workloads (no reduced-precision tensor path).
+// One warp per query row, 32 keys at a time: lane j scores key j of the chunk
+// over the whole head dimension (its K row loads in flight with the other
+// lanes'), the warp folds the chunk into the running softmax, and each lane
+// accumulates P V for D/32 output columns.  Exact fp32 math for the fp32
+// workloads (no reduced-precision tensor path).
 template <int D>
 __global__ void __launch_bounds__(128) attn_f32_kernel(const AttnParams p) {
   constexpr int kPer = D / 32;
@@ -535,6 +538,7 @@ __global__ void __launch_bounds__(128) attn_f32_kernel(const AttnParams p) {
   __shared__ float s_lse[kRowsPerCta];
   __shared__ int s_par[kMaxNodes];
   __shared__ uint64_t s_anc[kMaxNodes][2];
+  __shared__ __align__(16) float s_q[4][D];          // each warp's current query row
   float* s_o = reinterpret_cast<float*>(smem_raw);   // [64][D] split output rows
   pdl_launch_dependents();
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -562,64 +566,93 @@ __global__ void __launch_bounds__(128) attn_f32_kernel(const AttnParams p) {
   const int ntree_keys = kr.ntree > 0 ? n : 0;
   if (ntree_keys) tree_ancestors(p.parent, s0, n, s_par, s_anc);
 
+  // element offset of key t's K / V row for this (sequence, KV head), or -1
+  // when the key does not take part (not an ancestor, or a bad page)
+  auto key_off = [&](int t, uint64_t alo, uint64_t ahi) -> long long {
+    if (t >= nctx_keys) {
+      const int key = t - nctx_keys;
+      if (!anc_bit(alo, ahi, key)) return -1;
+      return (static_cast<long long>(s0 + key) * p.Hkv + g) * D;
+    }
+    const int key = kr.kbeg + t;
+    if (ps == 0) return ((static_cast<long long>(b) * p.Hkv + g) * p.ctx_max + key) * D;
+    const int page = p.page_table[static_cast<size_t>(b) * p.pages_per_seq + key / ps];
+    if (page < 0 || page >= p.num_pages) {
+      set_status(p.status, ASD_ERR_CTX_RANGE);
+      return -1;
+    }
+    return ((static_cast<long long>(page) * p.Hkv + g) * ps + key % ps) * D;
+  };
+  const int nkeys = nctx_keys + ntree_keys;
+  float* s_qw = s_q[warp];
+
   for (int r = warp; r < nrows; r += 4) {
     const size_t gr = rm.grow(r);
-    if (nctx_keys + ntree_keys == 0) {
+    if (nkeys == 0) {
       // empty split: weight-zero log-sum-exp and a finite (zero) row
       if (lane == 0) s_lse[r] = -INFINITY;
 #pragma unroll
       for (int k = 0; k < kPer; ++k) s_o[r * D + lane + 32 * k] = 0.f;
       continue;
     }
-    float qv[kPer], ov[kPer];
+    __syncwarp();
 #pragma unroll
-    for (int k = 0; k < kPer; ++k) {
-      qv[k] = qp[gr * D + lane + 32 * k];
-      ov[k] = 0.f;
-    }
+    for (int k = 0; k < kPer; ++k) s_qw[lane + 32 * k] = qp[gr * D + lane + 32 * k];
+    __syncwarp();
     uint64_t alo = 0, ahi = 0;
     if (ntree_keys) {
       const int node = (r0 + r) / p.G;
       alo = s_anc[node][0];
       ahi = s_anc[node][1];
     }
+    float ov[kPer];
+#pragma unroll
+    for (int k = 0; k < kPer; ++k) ov[k] = 0.f;
     float m = -INFINITY, l = 0.f;
-    for (int t = 0; t < nctx_keys + ntree_keys; ++t) {
-      const float* kr_;
-      const float* vr;
-      if (t >= nctx_keys) {
-        const int key = t - nctx_keys;
-        if (!anc_bit(alo, ahi, key)) continue;
-        const size_t off = (static_cast<size_t>(s0 + key) * p.Hkv + g) * D;
-        kr_ = tk + off;
-        vr = tv + off;
-      } else if (ps == 0) {
-        const int key = kr.kbeg + t;
-        const size_t off = ((static_cast<size_t>(b) * p.Hkv + g) * p.ctx_max + key) * D;
-        kr_ = kc + off;
-        vr = vc + off;
-      } else {
-        const int key = kr.kbeg + t;
-        const int page = p.page_table[static_cast<size_t>(b) * p.pages_per_seq + key / ps];
-        if (page < 0 || page >= p.num_pages) {
-          if (lane == 0) set_status(p.status, ASD_ERR_CTX_RANGE);
-          continue;
+    // 32 keys at a time: lane j scores key t0 + j over the whole head
+    // dimension, then the warp folds the chunk into the running softmax and
+    // every lane adds p_j V_j to its D/32 output columns
+    for (int t0 = 0; t0 < nkeys; t0 += 32) {
+      const int t = t0 + lane;
+      const long long off = t < nkeys ? key_off(t, alo, ahi) : -1;
+      float dot = -INFINITY;
+      if (off >= 0) {
+        const float4* kr4 = reinterpret_cast<const float4*>((t >= nctx_keys ? tk : kc) + off);
+        const float4* q4 = reinterpret_cast<const float4*>(s_qw);
+        float acc = 0.f;
+#pragma unroll 8
+        for (int d = 0; d < D / 4; ++d) {
+          const float4 kk = kr4[d], qq = q4[d];
+          acc = fmaf(qq.x, kk.x, acc);
+          acc = fmaf(qq.y, kk.y, acc);
+          acc = fmaf(qq.z, kk.z, acc);
+          acc = fmaf(qq.w, kk.w, acc);
         }
-        const size_t off = ((static_cast<size_t>(page) * p.Hkv + g) * ps + key % ps) * D;
-        kr_ = kc + off;
-        vr = vc + off;
+        dot = acc;
       }
-      float dot = 0.f;
+      float cm = dot;
 #pragma unroll
-      for (int k = 0; k < kPer; ++k) dot = fmaf(qv[k], kr_[lane + 32 * k], dot);
+      for (int o = 16; o > 0; o >>= 1) cm = fmaxf(cm, __shfl_xor_sync(0xffffffffu, cm, o));
+      if (cm == -INFINITY) continue;          // nothing visible in this chunk (uniform)
+      const float mn = fmaxf(m, cm);
+      const float al = m == -INFINITY ? 0.f : exp2f((m - mn) * c);
+      const float pe = dot == -INFINITY ? 0.f : exp2f((dot - mn) * c);
+      float ps_ = pe;
 #pragma unroll
-      for (int off = 16; off > 0; off >>= 1) dot += __shfl_xor_sync(0xffffffffu, dot, off);
-      const float mn = fmaxf(m, dot);
-      const float al = exp2f((m - mn) * c);
-      const float pe = exp2f((dot - mn) * c);
-      l = l * al + pe;
+      for (int o = 16; o > 0; o >>= 1) ps_ += __shfl_xor_sync(0xffffffffu, ps_, o);
+      l = l * al + ps_;
 #pragma unroll
-      for (int k = 0; k < kPer; ++k) ov[k] = fmaf(pe, vr[lane + 32 * k], ov[k] * al);
+      for (int k = 0; k < kPer; ++k) ov[k] *= al;
+      const int nj = min(32, nkeys - t0);
+#pragma unroll 4
+      for (int j = 0; j < nj; ++j) {
+        const float pj = __shfl_sync(0xffffffffu, pe, j);
+        const long long oj = __shfl_sync(0xffffffffu, off, j);
+        if (pj == 0.f || oj < 0) continue;    // uniform over the warp
+        const float* vr = (t0 + j >= nctx_keys ? tv : vc) + oj;
+#pragma unroll
+        for (int k = 0; k < kPer; ++k) ov[k] = fmaf(pj, vr[lane + 32 * k], ov[k]);
+      }
       m = mn;
     }
     const float inv = l > 0.f ? 1.f / l : 0.f;
