@@ -167,6 +167,7 @@ class Clocks:
     def __init__(self, gpu_index, enabled=True):
         self.proc = None
         self.path = None
+        self.gpu_index = gpu_index
         if not enabled:
             return
         fd, self.path = tempfile.mkstemp(suffix=".csv")
@@ -193,14 +194,28 @@ class Clocks:
                 if len(r) >= 9:
                     rows.append([x.strip() for x in r])
         os.unlink(self.path)
+        note = None
+        if not rows:
+            # a timed region shorter than the sampling interval: one sample at its end
+            try:
+                out = subprocess.run(["nvidia-smi", "-i", str(self.gpu_index),
+                                      f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits"],
+                                     capture_output=True, text=True, timeout=10).stdout
+                rows = [[x.strip() for x in r] for r in csv.reader(out.splitlines()) if len(r) >= 9]
+                note = "timed region shorter than the 200 ms sampling interval: one sample at its end"
+            except Exception:
+                rows = []
         if not rows:
             return None
         sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
         mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
         reasons = sorted({n for r in rows for n, v in zip(names, r[5:9]) if v.lower() == "active"})
-        return {"sm_mhz": statistics.median(sm) if sm else None,
-                "sm_max_mhz": max(mx) if mx else None, "reasons": reasons, "samples": len(rows)}
+        res = {"sm_mhz": statistics.median(sm) if sm else None,
+               "sm_max_mhz": max(mx) if mx else None, "reasons": reasons, "samples": len(rows)}
+        if note:
+            res["note"] = note
+        return res
 
 
 def slowest_rank(values, world, device):
@@ -499,7 +514,7 @@ def run_asd(args):
                        "peak": tpk, "unit": "TFLOP/s", "frac": tf / tpk,
                        "peak_source": tpk_kind + " bf16_tflops (MEASURED_PEAKS.json)",
                        "algorithmic_flops_per_launch": lm_flops, "avg_launch_us": 1e3 * lm_ms,
-                       "traffic": None}
+                       "traffic": LMHEAD_TRAFFIC_BY_CONFIG.get(CONFIG) if packed and not lazy else None}
     line = {
         "metric": METRIC, "value": job_value(wl.T, world, ms * 1e-3), "unit": UNIT, "n_gpus": world,
         "steps": K, "warmup": W, "ms_per_step": ms, "us_per_step": 1e3 * ms,
