@@ -81,8 +81,12 @@ def _run(dev, wl, tau, packed):
     return out, step.device_status()
 
 
-@pytest.mark.parametrize("cfg,over", [(2, None), (3, None), (4, None), (5, None), (2, dict(D=64))])
+@pytest.mark.parametrize("cfg,over", [(2, None), (3, None), (4, None), (5, None), (2, dict(D=64)),
+                                      (5, dict(B=8)), (5, dict(B=9))])
 def test_packed_verify_step_is_bit_identical(dev, cfg, over):
+    """Both weight layouts give the same bits; B = 8, 9 at 128 nodes each run
+    the LM head in clusters of two (multicast of the packed copies, an odd
+    number of node pairs for B = 9)."""
     wl = H.prepared(cfg, small=True, overrides=over)
     tau = 0.3
     rows, s0 = _run(dev, wl, tau, packed=False)
