@@ -2,10 +2,12 @@
 
 The translation units compile in parallel; the shared library links the CUDA
 runtime dynamically so that it shares the runtime instance already loaded by
-PyTorch.  Re-running is cheap: nothing is rebuilt when the library is newer
-than every source and header.
+PyTorch.  Re-running is cheap: nothing is rebuilt while the hash of the
+sources, the header and the build settings matches the one stored with the
+library.
 """
 import concurrent.futures
+import hashlib
 import os
 import shutil
 import subprocess
@@ -17,6 +19,7 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 OUT_DIR = os.path.join(HERE, "_lib")
 LIB_PATH = os.path.join(OUT_DIR, "libasd.so")
+HASH_PATH = os.path.join(OUT_DIR, "libasd.sha256")
 UNITS = ["tree_prep", "attention", "attention_tc", "lmhead_tc", "lmhead_f32", "tail", "asd_api", "policy", "lazy"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
@@ -38,11 +41,23 @@ def _sources():
     return deps
 
 
+def _digest() -> str:
+    """Hash of every source, the header and the build settings: the library is
+    rebuilt whenever any of them changes, whatever the files' timestamps."""
+    h = hashlib.sha256()
+    h.update(repr((UNITS, ARCH)).encode())
+    for f in sorted(_sources()):
+        h.update(os.path.basename(f).encode())
+        with open(f, "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()
+
+
 def up_to_date() -> bool:
-    if not os.path.exists(LIB_PATH):
+    if not (os.path.exists(LIB_PATH) and os.path.exists(HASH_PATH)):
         return False
-    t = os.path.getmtime(LIB_PATH)
-    return all(os.path.getmtime(f) < t for f in _sources())
+    with open(HASH_PATH) as fh:
+        return fh.read().strip() == _digest()
 
 
 def build(force: bool = False, verbose: bool = False) -> str:
@@ -74,6 +89,8 @@ def build(force: bool = False, verbose: bool = False) -> str:
     if r.returncode != 0:
         raise RuntimeError(f"link failed:\n{r.stdout}\n{r.stderr}")
     os.replace(tmp, LIB_PATH)
+    with open(HASH_PATH, "w") as fh:
+        fh.write(_digest())
     return LIB_PATH
 
 
