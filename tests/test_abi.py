@@ -165,3 +165,54 @@ def test_lm_schedule_host_checks(lib):
         assert fn(ctypes.byref(d), buf, buf, buf, buf, buf, 8, ctypes.c_float(0.5), *([buf] * 6),
                   buf, 1 << 20, None) == 2
         assert lib.asd_workspace_bytes(ctypes.byref(d), 8) == 0
+
+
+def _struct_members(src, name):
+    """Member names, in order, of `typedef struct name {...} name;` in asd.h."""
+    body = re.search(r"typedef struct " + name + r" \{(.*?)\} " + name + ";", src, re.S).group(1)
+    body = re.sub(r"/\*.*?\*/", "", body, flags=re.S)
+    names = []
+    for decl in body.split(";"):
+        m = re.search(r"(\w+)\s*(\[[^\]]*\])?\s*$", decl.strip())
+        if m and decl.strip():
+            names.append(m.group(1))
+    return names
+
+
+def _enum_values(src, name):
+    body = re.search(r"typedef enum " + name + r" \{(.*?)\} " + name + ";", src, re.S).group(1)
+    body = re.sub(r"/\*.*?\*/", "", body, flags=re.S)
+    return {k: int(v) for k, v in re.findall(r"(\w+)\s*=\s*(-?\d+)", body)}
+
+
+def test_binding_structs_and_constants_match_header():
+    """The ctypes structs carry the header's members in the header's order,
+    their sizes are those of the C layout, and the binding's constants equal
+    the header's enumerators."""
+    import ctypes
+    from paper_2609_02897_gb300 import build
+    build.build()
+    from paper_2609_02897_gb300 import asd
+    src = open(os.path.join(ROOT, "include", "asd.h")).read()
+    assert _struct_members(src, "asd_dims") == [f for f, _ in asd.Dims._fields_]
+    assert ctypes.sizeof(asd.Dims) == 4 * len(asd.Dims._fields_)
+    assert _struct_members(src, "asd_verify_args") == [f for f, _ in asd.VerifyArgs._fields_]
+    assert _struct_members(src, "asd_policy_params") == [f for f, _ in asd.PolicyParams._fields_]
+    assert ctypes.sizeof(asd.PolicyParams) == 3 * 8 + 8 * 4
+    assert _struct_members(src, "asd_policy_state") == ["rar", "zero_streak", "breaks"]
+    assert asd.POLICY_STATE_BYTES == 16
+    st = _enum_values(src, "asd_status")
+    assert {v: k for k, v in st.items()} == asd.STATUS
+    assert _enum_values(src, "asd_dtype") == {"ASD_F32": asd.ASD_F32, "ASD_BF16": asd.ASD_BF16}
+    assert _enum_values(src, "asd_accept_rule") == {
+        "ASD_ACCEPT_LONGEST": asd.ASD_ACCEPT_LONGEST, "ASD_ACCEPT_ONCE": asd.ASD_ACCEPT_ONCE,
+        "ASD_ACCEPT_GREEDY": asd.ASD_ACCEPT_GREEDY,
+        "ASD_ACCEPT_GREEDY_ONCE": asd.ASD_ACCEPT_GREEDY_ONCE}
+    assert _enum_values(src, "asd_lm_layout") == {"ASD_LM_ROWS": asd.ASD_LM_ROWS,
+                                                  "ASD_LM_PACKED": asd.ASD_LM_PACKED}
+    assert _enum_values(src, "asd_lm_schedule") == {
+        "ASD_LM_EVERY_ROW": asd.ASD_LM_EVERY_ROW, "ASD_LM_LAZY_LEVELS": asd.ASD_LM_LAZY_LEVELS}
+    defines = dict(re.findall(r"#define (ASD_\w+) \(?(\d+)", src))
+    assert int(defines["ASD_MAX_TREE_NODES"]) == asd.MAX_TREE_NODES
+    assert int(defines["ASD_NUM_STAGE_EVENTS"]) == asd.NUM_STAGE_EVENTS
+    assert int(defines["ASD_ABI_VERSION"]) == asd.abi_version()
