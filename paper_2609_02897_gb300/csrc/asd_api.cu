@@ -626,9 +626,11 @@ asd_status asd_verify_step(const asd_dims* dims, const asd_verify_args* a, void*
     return ASD_ERR_CUDA;
   record(a->stage_events[1], c.st);
   // The LM head goes first and takes one CTA per SM; the attention kernel
-  // starts right behind it (it reads no output of the LM head) and its CTAs
-  // share the SMs with the LM head's while the weights stream in.  The lazy
-  // schedule also finalises the rows it computes, so the tail only walks.
+  // starts right behind it (it reads no output of the LM head).  Up to 128
+  // nodes its CTAs share the SMs with the LM head's while the weights stream
+  // in; beyond that the wide LM head fills the SMs' shared memory and the
+  // tensor-core attention runs after it.  The lazy schedule also finalises
+  // the rows it computes, so the tail only walks.
   const bool lazy = c.d.lm_head_schedule == ASD_LM_LAZY_LEVELS;
   st = lazy ? run_lmhead_lazy(c, a->hidden, a->w_lm, a->parent, a->tokens, a->cu_nodes, a->tau,
                               a->row_max, a->row_argmax, a->row_lse, a->l_draft, a->ratio,

@@ -1,5 +1,7 @@
 // Tree attention of the verify pass (Sec. 2 "Verify": the target scores every
-// drafted node of the tree in one forward pass).
+// drafted node of the tree in one forward pass): the bf16 kernel that shares
+// the SMs with the LM head (steps of up to 128 nodes; more go to the
+// tensor-core kernel in attention_tc.cu) and the exact fp32 kernel.
 //
 // Work unit: one CTA per (row block, sequence x KV head, context split).  The
 // query rows of a (sequence, KV head) pair are its N nodes times the G query
