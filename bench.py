@@ -539,7 +539,8 @@ def run_asd(args):
                       "step_with_stage_events": 1e3 * staged_ms,
                       "note": "second timed region with events between kernels (no overlap)"},
         "mean_path_len": mean_path,
-        "gpu_launches": K * (N_STAGE_KERNELS + (1 + 2 * wl.max_path - 1 if lazy else 0)),
+        # every rank's launches in the timed region (the whole job, like `value`)
+        "gpu_launches": world * K * (N_STAGE_KERNELS + (1 + 2 * wl.max_path - 1 if lazy else 0)),
         "clocks": clk,
         "e2e": e2e,
     }
