@@ -311,6 +311,9 @@ int32_t asd_abi_version(void);
  * nothing.
  *  - The first call on a device, with that device current, looks up the
  *    array's device address; make that first call before any stream capture.
+ *    A device reset (cudaDeviceReset) gives the device a new context; the
+ *    first call after it looks the address up again, and should likewise
+ *    precede any capture.
  *  - Requests whose scratch needs exceed ASD_NOALLOC_SCRATCH_BYTES return
  *    ASD_ERR_WORKSPACE without enqueuing anything (about 3,400 tree nodes on a
  *    152-SM GB300: the scratch holds 16 bytes per node per SM plus 32 bytes

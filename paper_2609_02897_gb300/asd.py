@@ -24,6 +24,7 @@ ASD_LM_ROWS, ASD_LM_PACKED = 0, 1
 ASD_ACCEPT_LONGEST, ASD_ACCEPT_ONCE, ASD_ACCEPT_GREEDY, ASD_ACCEPT_GREEDY_ONCE = 0, 1, 2, 3
 ASD_LM_EVERY_ROW, ASD_LM_LAZY_LEVELS = 0, 1
 MAX_TREE_NODES = 128
+NOALLOC_SCRATCH_BYTES = 8 << 20   # ASD_NOALLOC_SCRATCH_BYTES
 NUM_STAGE_EVENTS = 5
 STATUS = {0: "ASD_OK", 1: "ASD_ERR_INVALID_ARG", 2: "ASD_ERR_SHAPE", 3: "ASD_ERR_TREE",
           4: "ASD_ERR_TOKEN_RANGE", 5: "ASD_ERR_CTX_RANGE", 6: "ASD_ERR_WORKSPACE",

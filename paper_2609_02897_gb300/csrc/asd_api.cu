@@ -696,37 +696,52 @@ static __device__ __align__(256) uint8_t g_noalloc_scratch[ASD_NOALLOC_SCRATCH_B
 
 namespace {
 
-std::mutex g_noalloc_mutex;
-void* g_noalloc_ptr[128] = {nullptr};
+typedef CUresult (*CtxGetCurrentFn)(CUcontext*);
 
-// Device address of the scratch array on the current device; set up on the
-// first call per device (this first call must precede any stream capture).
+CtxGetCurrentFn ctx_get_current_fn() {
+  static CtxGetCurrentFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &ptr, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<CtxGetCurrentFn>(ptr);
+  });
+  return fn;
+}
+
+std::mutex g_noalloc_mutex;
+struct NoallocSlot {
+  CUcontext ctx;
+  void* ptr;
+};
+NoallocSlot g_noalloc[128] = {};
+
+// Device address of the scratch array on the current device.  It is looked
+// up with the device current on the first call in each context of the device
+// (this first call must precede any stream capture); a device reset creates
+// a new context, so the next call looks the address up again.
 void* noalloc_scratch() {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 128) return nullptr;
+  CtxGetCurrentFn get = ctx_get_current_fn();
+  if (!get) return nullptr;
+  CUcontext ctx = nullptr;
+  if (get(&ctx) != CUDA_SUCCESS) return nullptr;
   std::lock_guard<std::mutex> lock(g_noalloc_mutex);
-  if (!g_noalloc_ptr[dev]) {
+  NoallocSlot& slot = g_noalloc[dev];
+  if (!ctx || !slot.ptr || slot.ctx != ctx) {
+    // the lookup also makes the device's primary context current if no
+    // runtime call has done so yet
     void* p = nullptr;
-    if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess) return nullptr;
-    g_noalloc_ptr[dev] = p;
+    if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p) return nullptr;
+    if (get(&ctx) != CUDA_SUCCESS || !ctx) return nullptr;
+    slot.ctx = ctx;
+    slot.ptr = p;
   }
-  return g_noalloc_ptr[dev];
-}
-
-// Regions of the LM-head path only (no attention partials).
-WsLayout lmhead_only_layout(const asd_dims& d, int T, int nsm) {
-  WsLayout L{};
-  L.g_lm = lm_ranges(d.vocab, nsm);
-  size_t off = 0;
-  L.status = off;      off = align256(off + 16);
-  L.seq_flags = off;   off = align256(off + 4 * static_cast<size_t>(d.batch));
-  L.child_start = off; off = align256(off + 4 * static_cast<size_t>(T));
-  L.child_cnt = off;   off = align256(off + 4 * static_cast<size_t>(T));
-  L.child_tok = off;   off = align256(off + 4 * static_cast<size_t>(T));
-  L.child_id = off;    off = align256(off + 4 * static_cast<size_t>(T));
-  L.lm_part = off;     off = align256(off + sizeof(LmPartial) * static_cast<size_t>(T) * L.g_lm);
-  L.total = off;
-  return L;
+  return slot.ptr;
 }
 
 }  // namespace
@@ -749,7 +764,9 @@ extern "C" asd_status asd_lmhead_margin_noalloc(
   Ctx c;
   c.d = *dims;
   c.T = total_nodes;
-  c.L = lmhead_only_layout(*dims, total_nodes, nsm);
+  // the every-row schedule's workspace regions (status, flags, children lists,
+  // LM-head partials), as asd_workspace_bytes counts them
+  c.L = layout(*dims, total_nodes, nsm);
   if (c.L.total > ASD_NOALLOC_SCRATCH_BYTES) return ASD_ERR_WORKSPACE;
   c.ws = noalloc_scratch();
   if (!c.ws) return ASD_ERR_CUDA;

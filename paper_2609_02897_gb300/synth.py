@@ -74,19 +74,34 @@ P_RANK2TO5 = 0.3  # drafted token = one of the parent row's rank-2..5 tokens
 # remainder (0.2): uniform over the vocabulary
 
 
+_ROUND_CHUNK = 1 << 16
+
+
+def _round_bf16_inplace(x: np.ndarray) -> np.ndarray:
+    """Rounds a contiguous float32 array to bfloat16 values in place, in
+    cache-sized chunks of 32-bit integer arithmetic (the sum wraps modulo 2^32
+    only for NaN patterns, which then end as the wider computation's would)."""
+    u = x.reshape(-1).view(np.uint32)
+    for i in range(0, u.size, _ROUND_CHUNK):
+        c = u[i:i + _ROUND_CHUNK]
+        t = c >> 16
+        t &= 1
+        t += 0x7FFF
+        c += t
+        c &= np.uint32(0xFFFF0000)
+    return x
+
+
 def round_bf16(x: np.ndarray) -> np.ndarray:
     """Round float32 values to the nearest bfloat16 (ties to even); float32 out."""
-    x = np.ascontiguousarray(x, dtype=np.float32)
-    u = x.view(np.uint32).astype(np.uint64)
-    u = (u + 0x7FFF + ((u >> 16) & 1)) & 0xFFFF0000
-    return u.astype(np.uint32).view(np.float32)
+    return _round_bf16_inplace(np.array(x, dtype=np.float32, order="C", copy=True))
 
 
 def _normal(rng: np.random.Generator, shape, std: float, bf16: bool) -> np.ndarray:
     x = rng.standard_normal(shape, dtype=np.float32)
     if std != 1.0:
         x *= np.float32(std)
-    return round_bf16(x) if bf16 else x
+    return _round_bf16_inplace(x) if bf16 else x
 
 
 # --------------------------------------------------------------------------

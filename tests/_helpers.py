@@ -114,19 +114,46 @@ def valid_path(parent_local, accept_local, path):
     return len(path) == best
 
 
-def compare_verify(wl, tau, out, seqs=None, check_attn_nodes=None, rule=0):
+def reached_rows(wl, accept):
+    """Roots, and every node whose parent is reached and which is accepted: the
+    rows whose verdicts the accepted-path walk can need (a node is judged by its
+    parent's row, and every walk moves from the root through accepted nodes)."""
+    r = np.zeros(wl.T, bool)
+    for b in range(wl.B):
+        s, e = int(wl.cu_nodes[b]), int(wl.cu_nodes[b + 1])
+        r[s] = True
+        for i in range(s + 1, e):
+            r[i] = r[s + int(wl.parent[i])] and int(accept[i]) == 1
+    return r
+
+
+def compare_verify(wl, tau, out, seqs=None, check_attn_nodes=None, rule=0, lazy=False):
     """Compares one verify step's outputs (numpy copies in `out`) with the
     oracle on the sequences `seqs` (all by default), the committed path under
-    accepted-path reading `rule`.  Returns a Report."""
+    accepted-path reading `rule`.  Returns a Report.
+
+    lazy: the step ran the lazy LM-head schedule, which computes only the rows
+    of the roots and of the nodes reached through accepted nodes.  The rows it
+    computed must be exactly that set under its own verdicts; the oracle then
+    evaluates the same rows (Eq. 1 and the kappa rule on their children) and
+    every computed statistic and every judged verdict is compared as for the
+    every-row schedule.  Outside the reported band the verdicts agree, so the
+    reached sets agree too; the rest keeps the documented fills."""
     rep = Report()
     atol, rtol = tol(wl)
     B = wl.B
     seqs = list(range(B)) if seqs is None else list(seqs)
     nodes = np.concatenate([np.arange(wl.cu_nodes[b], wl.cu_nodes[b + 1]) for b in seqs])
     gp = wl.global_parent()
+    all_nodes = nodes
+    if lazy:
+        reach = ~np.isnan(out["row_max"])
+        np.testing.assert_array_equal(reach, reached_rows(wl, out["accept"]),
+                                      err_msg="lazy schedule: rows computed")
+        nodes = nodes[reach[nodes]]
 
     # step 1: attention
-    att_nodes = nodes if check_attn_nodes is None else np.asarray(check_attn_nodes)
+    att_nodes = all_nodes if check_attn_nodes is None else np.asarray(check_attn_nodes)
     ref_attn = oracle.tree_attention(wl.q, wl.k_cache, wl.v_cache, wl.ctx_len, wl.tree_k,
                                      wl.tree_v, wl.parent, wl.cu_nodes, wl.page_table,
                                      wl.page_size, nodes=att_nodes)
@@ -145,14 +172,27 @@ def compare_verify(wl, tau, out, seqs=None, check_attn_nodes=None, rule=0):
     for r in nodes:
         if int(r) not in tie:
             assert out["row_argmax"][r] == lm["row_argmax"][r], f"argmax row {r}"
-    kids = np.array([c for c in nodes if gp[c] >= 0], dtype=np.int64)
+    if lazy:
+        # judged nodes: those whose parent row was computed
+        judged = set(int(c) for c in all_nodes if gp[c] >= 0 and reach[gp[c]])
+        kids = np.array(sorted(judged), dtype=np.int64)
+        rest = np.array([c for c in all_nodes if gp[c] >= 0 and int(c) not in judged],
+                        dtype=np.int64)
+        if len(rest):
+            assert np.all(out["accept"][rest] == 0)
+            assert np.all(np.isnan(out["ratio"][rest])) and np.all(np.isnan(out["l_draft"][rest]))
+        unreached = all_nodes[~reach[all_nodes]]
+        assert np.all(np.isnan(out["row_lse"][unreached]))
+        assert np.all(out["row_argmax"][unreached] == -1)
+    else:
+        kids = np.array([c for c in nodes if gp[c] >= 0], dtype=np.int64)
     if len(kids):
         rep.max_err["l_draft"] = assert_close(out["l_draft"][kids], lm["l_draft"][kids], atol, rtol,
                                               "l_draft")
         rep.max_err["ratio"] = assert_close(out["ratio"][kids], lm["ratio"][kids], 1e-6, 5e-2,
                                             "ratio")
         assert np.all(out["ratio"][kids] <= 1.0) and np.all(out["ratio"][kids] >= 0.0)
-    roots = np.array([c for c in nodes if gp[c] < 0])
+    roots = np.array([c for c in all_nodes if gp[c] < 0])
     assert np.all(out["accept"][roots] == 1)
     band = set()
     for c in kids:
@@ -167,7 +207,7 @@ def compare_verify(wl, tau, out, seqs=None, check_attn_nodes=None, rule=0):
         # the greedy walks order promoted siblings by ratio: near-equal ratios
         # cannot be ordered alike in fp32 and fp64
         for u in nodes:
-            sib = sorted((float(lm["ratio"][c]) for c in kids if gp[c] == u and lm["accept"][c]
+            sib = sorted((float(lm["ratio"][c]) for c in kids if gp[c] == u and lm["accept"][c] == 1
                           and int(wl.tokens[c]) != int(lm["row_argmax"][u])), reverse=True)
             if len(sib) > 1 and sib[0] - sib[1] < 1e-3:
                 band.update(int(c) for c in kids if gp[c] == u)

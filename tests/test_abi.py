@@ -216,3 +216,5 @@ def test_binding_structs_and_constants_match_header():
     assert int(defines["ASD_MAX_TREE_NODES"]) == asd.MAX_TREE_NODES
     assert int(defines["ASD_NUM_STAGE_EVENTS"]) == asd.NUM_STAGE_EVENTS
     assert int(defines["ASD_ABI_VERSION"]) == asd.abi_version()
+    m = re.search(r"#define ASD_NOALLOC_SCRATCH_BYTES \((\d+)u << (\d+)\)", src)
+    assert m and int(m.group(1)) << int(m.group(2)) == asd.NOALLOC_SCRATCH_BYTES

@@ -77,11 +77,16 @@ def test_noalloc_rejects_requests_larger_than_its_scratch():
     wl = H.prepared(2, small=True)
     d = _device.to_device(wl)
     dims = _device.dims_of(wl)
-    # 40 trees of 128 nodes need ~12 MB of scratch on a 152-SM GPU (limit 8 MiB)
-    dims.batch = 40
+    # enough trees of 128 nodes that the scratch need (16 bytes per node per
+    # LM-head range, one range per SM up to the vocabulary's 32-row groups,
+    # plus the children lists) exceeds the limit on this GPU, whatever its SM count
     dims.max_nodes = 128
-    big = torch.zeros(40 * 128, dtype=torch.int32, device="cuda")
-    out = _outputs(40 * 128)
+    dims.batch = 1
+    while asd.asd_workspace_bytes(dims, dims.batch * 128) <= asd.NOALLOC_SCRATCH_BYTES:
+        dims.batch += 1
+    T = dims.batch * 128
+    big = torch.zeros(T, dtype=torch.int32, device="cuda")
+    out = _outputs(T)
     with pytest.raises(asd.AsdError) as e:
         asd.asd_lmhead_margin_noalloc(dims, d["hidden"], d["w_lm"], big, big, big, 0.3,
                                       out["row_max"], out["row_argmax"], out["row_lse"],
