@@ -135,7 +135,8 @@ __device__ __forceinline__ size_t grow_of(const AttnParams& p, const Item& it, i
   return static_cast<size_t>(it.s0 + i) * p.Hq + it.g * p.G + (rr - i * p.G);
 }
 
-// Issues the K and V tiles of tile t into one stage (producer lane only).
+// Issues the K and V tiles of a contiguous-cache or tree tile t into one
+// stage (producer lane 0 only).
 template <int D>
 __device__ __forceinline__ void issue_tile(const AttnParams& p, const Item& it, int t,
                                            uint32_t k_s, uint32_t v_s, uint32_t bar,
@@ -143,10 +144,10 @@ __device__ __forceinline__ void issue_tile(const AttnParams& p, const Item& it, 
                                            const CUtensorMap* tm_tk, const CUtensorMap* tm_tv,
                                            uint64_t pol) {
   using G = TcGeom<D>;
+  mbar_expect_tx(bar, 2 * G::kTileBytes);
   if (t >= it.nctx) {
     // tree keys: rows s0 + key0 .. of KV head g (rows past T read as zeros)
     const int key0 = (t - it.nctx) * kKeys;
-    mbar_expect_tx(bar, 2 * G::kTileBytes);
 #pragma unroll
     for (int h = 0; h < G::kNH; ++h) {
       tma_load_3d(k_s + h * (kKeys * 128), tm_tk, bar, h * 64, it.g, it.s0 + key0, pol);
@@ -154,44 +155,66 @@ __device__ __forceinline__ void issue_tile(const AttnParams& p, const Item& it, 
     }
     return;
   }
-  const int key0 = t * kKeys;
-  if (p.page_size == 0) {
-    const int row = (it.b * p.Hkv + it.g) * p.ctx_max + key0;
-    mbar_expect_tx(bar, 2 * G::kTileBytes);
+  const int row = (it.b * p.Hkv + it.g) * p.ctx_max + t * kKeys;
 #pragma unroll
-    for (int h = 0; h < G::kNH; ++h) {
-      tma_load_2d(k_s + h * (kKeys * 128), tm_k, bar, h * 64, row, pol);
-      tma_load_2d(v_s + h * (kKeys * 128), tm_v, bar, h * 64, row, pol);
-    }
-    return;
+  for (int h = 0; h < G::kNH; ++h) {
+    tma_load_2d(k_s + h * (kKeys * 128), tm_k, bar, h * 64, row, pol);
+    tma_load_2d(v_s + h * (kKeys * 128), tm_v, bar, h * 64, row, pol);
   }
-  // paged: one box of min(page, 128) rows per page the tile touches
+}
+
+constexpr int kPageChunk = 512;   // page-table entries staged in shared memory
+
+// Issues the K and V boxes of paged context tile t into one stage (the whole
+// producer warp): one box of min(page, 128) rows per page the tile touches,
+// lane j taking page j of the tile, its page id read from a chunk of the
+// sequence's page-table row that the warp stages in shared memory (`chunk0`:
+// first staged entry, -1 before the first chunk).  Pages past the context
+// are not loaded; an out-of-range page id is reported and not loaded.
+template <int D>
+__device__ __forceinline__ void issue_paged_tile(const AttnParams& p, const Item& it, int t,
+                                                 uint32_t k_s, uint32_t v_s, uint32_t bar,
+                                                 const CUtensorMap* tm_k, const CUtensorMap* tm_v,
+                                                 uint64_t pol, int* s_pages, int& chunk0,
+                                                 int lane) {
+  using G = TcGeom<D>;
   const int ps = p.page_size;
   const int br = ps < kKeys ? ps : kKeys;
-  const int nbox = kKeys / br;
-  int rows[kKeys / 8];
-  int cnt = 0;
-  for (int j = 0; j < nbox; ++j) {
-    const int key = key0 + j * br;
-    rows[j] = -1;
-    if (key >= it.ctx) continue;
-    const int page = p.page_table[static_cast<size_t>(it.b) * p.pages_per_seq + key / ps];
-    if (page < 0 || page >= p.num_pages) {
-      set_status(p.status, ASD_ERR_CTX_RANGE);
-      continue;
+  const int nbox = kKeys / br;   // <= 16 (pages hold at least 8 rows)
+  const int key0 = t * kKeys;
+  const int e_first = key0 / ps, e_last = (key0 + (nbox - 1) * br) / ps;
+  if (chunk0 < 0 || e_first < chunk0 || e_last >= chunk0 + kPageChunk) {
+    chunk0 = e_first;
+    const int32_t* row_pt = p.page_table + static_cast<size_t>(it.b) * p.pages_per_seq;
+    for (int i = lane; i < kPageChunk; i += 32) {
+      const int e = chunk0 + i;
+      s_pages[i] = e < p.pages_per_seq ? row_pt[e] : -1;
     }
-    rows[j] = (page * p.Hkv + it.g) * ps + (key % ps);
-    ++cnt;
+    __syncwarp();
   }
-  mbar_expect_tx(bar, static_cast<uint32_t>(cnt * 2 * G::kNH * br * 128));
-  for (int j = 0; j < nbox; ++j) {
-    if (rows[j] < 0) continue;
+  int row = -1;
+  if (lane < nbox) {
+    const int key = key0 + lane * br;
+    if (key < it.ctx) {
+      const int page = s_pages[key / ps - chunk0];
+      if (page < 0 || page >= p.num_pages)
+        set_status(p.status, ASD_ERR_CTX_RANGE);
+      else
+        row = (page * p.Hkv + it.g) * ps + (key % ps);
+    }
+  }
+  const uint32_t valid = __ballot_sync(0xffffffffu, row >= 0);
+  if (lane == 0)
+    mbar_expect_tx(bar, static_cast<uint32_t>(__popc(valid) * 2 * G::kNH * br * 128));
+  __syncwarp();
+  if (row >= 0) {
 #pragma unroll
     for (int h = 0; h < G::kNH; ++h) {
-      tma_load_2d(k_s + h * (kKeys * 128) + j * br * 128, tm_k, bar, h * 64, rows[j], pol);
-      tma_load_2d(v_s + h * (kKeys * 128) + j * br * 128, tm_v, bar, h * 64, rows[j], pol);
+      tma_load_2d(k_s + h * (kKeys * 128) + lane * br * 128, tm_k, bar, h * 64, row, pol);
+      tma_load_2d(v_s + h * (kKeys * 128) + lane * br * 128, tm_v, bar, h * 64, row, pol);
     }
   }
+  __syncwarp();
 }
 
 // Softmax warps (eight): warp w handles TMEM lane quarter w % 4 (its 32 query
@@ -376,6 +399,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   __shared__ uint64_t s_anc[kMaxNodes][2];
   __shared__ float s_mx[2][2][kRows];   // [tile parity][key half][row]: partial row max
   __shared__ float s_l[2][kRows];       // [key half][row]: partial row sum
+  __shared__ int s_pages[kPageChunk];   // producer: staged page-table entries (paged caches)
 
   pdl_launch_dependents();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -440,24 +464,34 @@ __global__ void __launch_bounds__(kThreads, 1)
       prefetch_tmap(&tm_v);
       prefetch_tmap(&tm_tk);
       prefetch_tmap(&tm_tv);
-      const uint64_t pol = l2_policy_evict_first();
-      int issued = 0;
-      for (int t = 0; t < it.ntiles; ++t) {
-        const int stage = t % kStages;
-        if (!mbar_wait(smem_u32(&s_kv_empty[stage]), ((t / kStages) & 1) ^ 1u)) {
+    }
+    const uint64_t pol = l2_policy_evict_first();
+    int issued = 0;
+    int chunk0 = -1;
+    for (int t = 0; t < it.ntiles; ++t) {
+      const int stage = t % kStages;
+      if (!wait_all(&s_kv_empty[stage], ((t / kStages) & 1) ^ 1u)) {
+        if (lane == 0) {
           set_status(p.status, ASD_ERR_TIMEOUT);
           s_abort = 1;
-          break;
         }
-        if (s_abort) break;
-        issue_tile<D>(p, it, t, k_s0 + stage * G::kTileBytes, v_s0 + stage * G::kTileBytes,
-                      smem_u32(&s_kv_full[stage]), &tm_k, &tm_v, &tm_tk, &tm_tv, pol);
-        ++issued;
+        break;
       }
-      // every copy issued has landed before the buffers are reused or left
+      if (aborted_warp(&s_abort)) break;
+      const uint32_t k_st = k_s0 + stage * G::kTileBytes, v_st = v_s0 + stage * G::kTileBytes;
+      if (p.page_size != 0 && t < it.nctx)
+        issue_paged_tile<D>(p, it, t, k_st, v_st, smem_u32(&s_kv_full[stage]), &tm_k, &tm_v, pol,
+                            s_pages, chunk0, lane);
+      else if (lane == 0)
+        issue_tile<D>(p, it, t, k_st, v_st, smem_u32(&s_kv_full[stage]), &tm_k, &tm_v, &tm_tk,
+                      &tm_tv, pol);
+      __syncwarp();
+      ++issued;
+    }
+    // every copy issued has landed before the buffers are reused or left
+    if (lane == 0)
       for (int t = max(0, issued - kStages); t < issued; ++t)
         mbar_wait(smem_u32(&s_kv_full[t % kStages]), (t / kStages) & 1);
-    }
     __syncwarp();
   } else if (warp == 1) {
     // --------------------------------------------------------------- MMA issuer
