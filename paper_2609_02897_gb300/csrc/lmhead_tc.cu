@@ -314,6 +314,12 @@ __global__ void __launch_bounds__(192, 1)
 // copying its half.  Every thread keeps one running state per vocabulary
 // range and writes one partial per range, so the statistics are those of
 // CTAs that own one range each, bit for bit.
+//
+// Warp roles (320 threads): warp 0 TMA producer, warp 1 TMEM allocator and MMA
+// issuer, warps 2-5 and 6-9 two epilogue groups; group g drains the
+// accumulator of the pair's node tile g, so that both accumulators of a
+// vocabulary tile are drained at once and the MMAs of the next tile wait for
+// one drain instead of two.
 constexpr int kWideN = 2 * kLmTileN;                 // vocabulary rows per MMA
 constexpr int kWideG = 2;                            // node tiles per W stage and CTA
 constexpr int kWideStages = 3;
@@ -321,6 +327,7 @@ constexpr int kWideA = kM * 128;                     // one node tile's k-block:
 constexpr int kWideSlot = kWideG * kWideA + kWideN * 128;   // 64 KB
 constexpr uint32_t kWideTmemCols = kWideG * kWideN;  // 512
 constexpr int kTileGroups = kLmTileN / kLmBoxRows;   // 32-row groups per packed tile
+constexpr int kWideThreads = 320;                    // producer, MMA, two epilogue groups
 
 __device__ __forceinline__ uint32_t cta_rank_in_cluster() {
   uint32_t r;
@@ -379,7 +386,7 @@ struct WideVocab {
 };
 
 template <int CL>
-__global__ void __launch_bounds__(192, 1)
+__global__ void __launch_bounds__(kWideThreads, 1)
     lmhead_wide_kernel(const __grid_constant__ LmMaps maps, const LmParams p) {
   extern __shared__ uint8_t smem_raw[];
   __shared__ __align__(8) uint64_t s_full[kWideStages];
@@ -631,40 +638,37 @@ __global__ void __launch_bounds__(192, 1)
     __syncwarp();
   } else {
     // ----------------------------------------------------------------- epilogue
-    // Thread `row` owns TMEM lane `row`: row `row` of both node tiles of the
-    // current pair, one running state per node tile and vocabulary range.
+    // Two groups of four warps: group g drains the accumulator of node tile
+    // j = g of the current pair, so both accumulators of a vocabulary tile
+    // drain at once.  Thread `row` of a group owns TMEM lane `row`: row `row`
+    // of its node tile, one running state per vocabulary range.
     const int q4 = warp & 3;
     const int row = q4 * 32 + lane;
+    const int g = (warp - 2) >> 2;
     pdl_wait();
     int used = 0;
     bool ok = true;
     for (int it = 0; it < nit && ok; ++it) {
       const int pi = it * CL + rank;
       const int gn = pi < nng ? min(kWideG, nnt - pi * kWideG) : 0;
-      RowState st[CL][kWideG];
-      bool act[kWideG];
+      const int r = (pi * kWideG + g) * kM + row;
+      const int node = (g < gn && r < nrow && p.row_node) ? p.row_node[r] : r;
+      const bool act = g < gn && r < nrow && node >= 0 && node < p.T;
+      RowState st[CL];
 #pragma unroll
-      for (int j = 0; j < kWideG; ++j) {
-        const int r = (pi * kWideG + j) * kM + row;
-        const int node = (j < gn && r < nrow && p.row_node) ? p.row_node[r] : r;
-        act[j] = j < gn && r < nrow && node >= 0 && node < p.T;
-#pragma unroll
-        for (int qq = 0; qq < CL; ++qq)
-          row_state_init(st[qq][j], act[j], node, (qq ? voc.gs1 : voc.gs0) * kLmBoxRows,
-                         p.child_start, p.child_cnt, p.child_tok, p.T);
-      }
+      for (int qq = 0; qq < CL; ++qq)
+        row_state_init(st[qq], act, node, (qq ? voc.gs1 : voc.gs0) * kLmBoxRows, p.child_start,
+                       p.child_cnt, p.child_tok, p.T);
       for (int vt = 0; vt < nvt && ok; ++vt) {
-#pragma unroll
-        for (int j = 0; j < kWideG; ++j) {
-          if (j >= gn || !ok) continue;
-          const int u = used + j;
+        if (g < gn) {
+          const int u = used + g;
           const int acc = u % kWideG;
           ok = __shfl_sync(0xffffffffu,
                            mbar_wait(smem_u32(&s_tfull[acc]), (static_cast<uint32_t>(u / kWideG)) & 1u),
                            0);
           if (!ok || s_abort) {
             ok = false;
-            continue;
+            break;
           }
           tc_fence_after();
           const uint32_t taddr = tmem + (static_cast<uint32_t>(q4 * 32) << 16) +
@@ -675,16 +679,23 @@ __global__ void __launch_bounds__(192, 1)
             if (2 * vt + hf >= voc.ntiles) break;
             int q, g0, ng, v0, rows;
             voc.tile(2 * vt + hf, p.V, q, g0, ng, v0, rows);
-            for (int c = 0; c < (rows + 31) / 32; ++c) {
-              float r[32];
-              tmem_ld32(taddr + hf * kLmTileN + 32 * c, r);
-              if (act[j]) {
-                if (CL == 2 && q == 1)
-                  row_chunk(st[CL - 1][j], r, v0 + 32 * c, min(32, rows - 32 * c), p.child_tok,
-                            p.child_id, p.l_draft, p.T);
-                else
-                  row_chunk(st[0][j], r, v0 + 32 * c, min(32, rows - 32 * c), p.child_tok,
-                            p.child_id, p.l_draft, p.T);
+            for (int c = 0; c < rows; c += 64) {
+              float x[64];
+              tmem_ld64(taddr + hf * kLmTileN + c, x);
+              if (act) {
+                float (&x0)[32] = *reinterpret_cast<float(*)[32]>(&x[0]);
+                float (&x1)[32] = *reinterpret_cast<float(*)[32]>(&x[32]);
+                const int n0 = min(32, rows - c), n1 = min(32, rows - c - 32);
+                if (CL == 2 && q == 1) {
+                  row_chunk(st[CL - 1], x0, v0 + c, n0, p.child_tok, p.child_id, p.l_draft, p.T);
+                  if (n1 > 0)
+                    row_chunk(st[CL - 1], x1, v0 + c + 32, n1, p.child_tok, p.child_id,
+                              p.l_draft, p.T);
+                } else {
+                  row_chunk(st[0], x0, v0 + c, n0, p.child_tok, p.child_id, p.l_draft, p.T);
+                  if (n1 > 0)
+                    row_chunk(st[0], x1, v0 + c + 32, n1, p.child_tok, p.child_id, p.l_draft, p.T);
+                }
               }
             }
           }
@@ -694,21 +705,15 @@ __global__ void __launch_bounds__(192, 1)
         }
         used += gn;
       }
-      if (ok) {
+      if (ok && g < gn && r < nrow) {   // partials by row, one per range
 #pragma unroll
-        for (int j = 0; j < kWideG; ++j) {
-          const int r = (pi * kWideG + j) * kM + row;   // partials by row, one per range
-          if (j < gn && r < nrow) {
-#pragma unroll
-            for (int qq = 0; qq < CL; ++qq) {
-              LmPartial part;
-              part.m = st[qq][j].m;
-              part.s = st[qq][j].s;
-              part.a = st[qq][j].a;
-              part.pad = 0;
-              p.part[static_cast<size_t>(r) * p.g_lm + cid * CL + qq] = part;
-            }
-          }
+        for (int qq = 0; qq < CL; ++qq) {
+          LmPartial part;
+          part.m = st[qq].m;
+          part.s = st[qq].s;
+          part.a = st[qq].a;
+          part.pad = 0;
+          p.part[static_cast<size_t>(r) * p.g_lm + cid * CL + qq] = part;
         }
       }
     }
@@ -794,7 +799,7 @@ cudaError_t launch_wide(const LmParams& p, const LmMaps& maps, cudaStream_t s) {
   if (err != cudaSuccess) return err;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(p.g_lm);
-  cfg.blockDim = dim3(192);
+  cfg.blockDim = dim3(kWideThreads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
   cudaLaunchAttribute attr[2];
