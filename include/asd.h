@@ -299,6 +299,21 @@ const char* asd_status_string(int32_t status);
 int32_t asd_abi_version(void);
 
 /*
+ * Test hook for the failure path (no counterpart in the paper).  Every wait
+ * of a kernel on its own pipeline (a TMA copy, an MMA, another warp) gives up
+ * after a bounded number of SM clock cycles, records ASD_ERR_TIMEOUT in the
+ * workspace status word, waits for the copies and MMAs it already started,
+ * releases its tensor memory and returns; the tail then commits nothing for
+ * any sequence of that call (path_len 0, ctx_len_out = ctx_len).  The bound
+ * is about 2 s of SM clocks.  This sets it, for the workspace-taking calls
+ * enqueued afterwards in this process, to `cycles` (0 restores the default)
+ * so that a test can make a wait give up on purpose; the waits for copies and
+ * MMAs already in flight keep the full bound.  Set it outside any stream
+ * capture.  Returns ASD_ERR_INVALID_ARG for a negative value.
+ */
+asd_status asd_debug_set_wait_cycles(int64_t cycles);
+
+/*
  * Allocation-free variant of asd_lmhead_margin (the paper has no counterpart;
  * this is a library convenience).  Same arguments and outputs, but instead
  * of a caller-provided workspace it uses scratch memory that the library

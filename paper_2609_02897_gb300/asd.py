@@ -33,7 +33,8 @@ EXPORTS = ["asd_workspace_bytes", "asd_tree_attention", "asd_lmhead_margin", "as
            "asd_kv_compact", "asd_verify_step", "asd_get_device_status", "asd_status_string",
            "asd_abi_version", "asd_lmhead_margin_noalloc", "asd_lm_head_packed_bytes",
            "asd_pack_lm_head",
-           "asd_policy_triplets", "asd_policy_init", "asd_policy_update", "asd_policy_select"]
+           "asd_policy_triplets", "asd_policy_init", "asd_policy_update", "asd_policy_select",
+           "asd_debug_set_wait_cycles"]
 
 
 class AsdError(RuntimeError):
@@ -108,6 +109,8 @@ _lib.asd_verify_step.argtypes = [_P, ctypes.POINTER(VerifyArgs), _vp, ctypes.c_s
 _lib.asd_lmhead_margin_noalloc.restype = ctypes.c_int
 _lib.asd_lmhead_margin_noalloc.argtypes = [_P] + [_vp] * 5 + [ctypes.c_int32, ctypes.c_float] + [
     _vp] * 6 + [_vp, _vp]
+_lib.asd_debug_set_wait_cycles.restype = ctypes.c_int
+_lib.asd_debug_set_wait_cycles.argtypes = [ctypes.c_int64]
 _lib.asd_get_device_status.restype = ctypes.c_int
 _lib.asd_get_device_status.argtypes = [_vp, ctypes.POINTER(ctypes.c_int32), _vp]
 _lib.asd_lm_head_packed_bytes.restype = ctypes.c_size_t
@@ -245,6 +248,12 @@ def asd_kv_compact(dims, tree_k, tree_v, cu_nodes, total_nodes, path, path_len, 
 def asd_verify_step(dims, args: VerifyArgs, workspace, stream=None):
     _check(_lib.asd_verify_step(ctypes.byref(dims), ctypes.byref(args), _ptr(workspace),
                                 workspace.numel(), _stream(stream)), "asd_verify_step")
+
+
+def asd_debug_set_wait_cycles(cycles: int):
+    """Test hook: the kernels' bounded waits give up after `cycles` SM clock
+    cycles in later calls (0 restores the default of about 2 s)."""
+    _check(_lib.asd_debug_set_wait_cycles(int(cycles)), "asd_debug_set_wait_cycles")
 
 
 def asd_get_device_status(workspace, stream=None) -> int:

@@ -1,6 +1,7 @@
 // C-ABI entry points of libasd (declared in include/asd.h): host-side argument
 // checks, workspace layout, TMA descriptors and kernel launches.  Nothing here
 // allocates device memory or synchronises, except asd_get_device_status.
+#include <atomic>
 #include <cmath>
 #include <cstring>
 #include <mutex>
@@ -172,6 +173,10 @@ struct Ctx {
   void* ws;
 };
 
+// Wait budget (SM clock cycles) that asd_debug_set_wait_cycles set for the
+// kernels of later calls; 0: the kernels' default.
+std::atomic<long long> g_wait_cycles{0};
+
 // Common checks of every workspace-taking call; fills ctx on success.
 asd_status begin_call(const asd_dims* dims, int32_t total_nodes, void* ws, size_t ws_bytes,
                       void* stream, Ctx* c) {
@@ -188,6 +193,12 @@ asd_status begin_call(const asd_dims* dims, int32_t total_nodes, void* ws, size_
   c->st = static_cast<cudaStream_t>(stream);
   c->ws = ws;
   if (cudaMemsetAsync(ws_at<int>(ws, c->L.status), 0, 16, c->st) != cudaSuccess)
+    return ASD_ERR_CUDA;
+  // a test's shorter wait budget rides in words 2-3 of the status block
+  static thread_local long long budget;
+  budget = g_wait_cycles.load();
+  if (budget != 0 && cudaMemcpyAsync(ws_at<int>(ws, c->L.status) + 2, &budget, sizeof(budget),
+                                     cudaMemcpyHostToDevice, c->st) != cudaSuccess)
     return ASD_ERR_CUDA;
   return ASD_OK;
 }
@@ -440,6 +451,12 @@ void record(void* ev, cudaStream_t st) {
 extern "C" {
 
 int32_t asd_abi_version(void) { return ASD_ABI_VERSION; }
+
+asd_status asd_debug_set_wait_cycles(int64_t cycles) {
+  if (cycles < 0) return ASD_ERR_INVALID_ARG;
+  g_wait_cycles.store(cycles);
+  return ASD_OK;
+}
 
 const char* asd_status_string(int32_t s) {
   switch (s) {

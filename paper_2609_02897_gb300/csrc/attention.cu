@@ -227,11 +227,13 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const __grid_constant__ 
                 "the K/V ring must hold the fp32 output rows");
   extern __shared__ uint8_t smem_raw[];
   __shared__ int s_abort;
+  __shared__ int s_abort_tile;   // the tile whose wait gave up
   __shared__ float s_lse[kRowsPerCta];
   __shared__ int s_par[kMaxNodes];
   __shared__ uint64_t s_anc[kMaxNodes][2];
 
   pdl_launch_dependents();  // nothing downstream reads this kernel's output early
+  const long long budget = wait_budget(p.status);
 
   // This kernel does not depend on the tree preparation: it derives the
   // ancestor masks itself and keeps every access inside the caller's arrays
@@ -400,10 +402,11 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const __grid_constant__ 
         *reinterpret_cast<uint4*>(gVs + sw_off<kKeysPerTile>(r, ch)) = vv;
       }
     } else {
-      const bool ok = mbar_wait(sBar + 8 * stage, (t / kAttnStages) & 1);
+      const bool ok = mbar_wait(sBar + 8 * stage, (t / kAttnStages) & 1, budget);
       if (!ok) {
-        set_status(p.status, ASD_ERR_TIMEOUT);
+        note_timeout(p.status);
         s_abort = 1;
+        s_abort_tile = t;
       } else if (valid < kKeysPerTile) {
         // rows past the context may hold anything: zero V so that 0 * V stays 0
         for (int cidx = tid; cidx < (kKeysPerTile - valid) * kChunks; cidx += 128) {
@@ -505,6 +508,12 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const __grid_constant__ 
   if (s_abort) {  // a bounded wait gave up: contribute nothing, still meet the cluster
     mA = mB = -INFINITY;
     lA = lB = 0.f;
+    // the tiles issued from the one that was not waited for on are still in
+    // flight: they land before the stage buffers serve the merge
+    if (tid == 0)
+      for (int tt = s_abort_tile; tt < kr.nctx && tt < s_abort_tile + kAttnStages; ++tt)
+        mbar_wait(sBar + 8 * (tt % kAttnStages), (tt / kAttnStages) & 1);
+    __syncthreads();
   }
 
   lA += __shfl_xor_sync(0xffffffffu, lA, 1);

@@ -95,9 +95,10 @@ __device__ __forceinline__ bool softmax_any(bool v) {
   return r != 0;
 }
 
-// Every lane polls (bounded); the result is lane 0's, uniform over the warp.
-__device__ __forceinline__ bool wait_all(uint64_t* bar, uint32_t parity) {
-  return __shfl_sync(0xffffffffu, mbar_wait(smem_u32(bar), parity) ? 1 : 0, 0) != 0;
+// Every lane polls (bounded by `budget` cycles); the result is lane 0's,
+// uniform over the warp.
+__device__ __forceinline__ bool wait_all(uint64_t* bar, uint32_t parity, long long budget) {
+  return __shfl_sync(0xffffffffu, mbar_wait(smem_u32(bar), parity, budget) ? 1 : 0, 0) != 0;
 }
 
 __device__ __forceinline__ bool aborted_warp(volatile int* s_abort) {
@@ -233,7 +234,8 @@ __device__ __forceinline__ bool softmax_role(const AttnParams& p, const Item& it
                                              float (*s_mx)[2][kRows], float (*s_l)[kRows],
                                              uint64_t* q_ready, uint64_t* s_full,
                                              uint64_t* p_full, uint64_t* pv_done,
-                                             volatile int* s_abort, float& inv) {
+                                             volatile int* s_abort, long long budget,
+                                             float& inv) {
   using G = TcGeom<D>;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int hf = (warp - 2) >> 2;              // key half of every tile
@@ -283,7 +285,7 @@ __device__ __forceinline__ bool softmax_role(const AttnParams& p, const Item& it
     const int valid = min(kKeys, (tree ? it.n : it.ctx) - key0);
     float x[64];
     float mt = -INFINITY;
-    const bool here = !bad && wait_all(&s_full[b], (t >> 1) & 1) && !aborted_warp(s_abort);
+    const bool here = !bad && wait_all(&s_full[b], (t >> 1) & 1, budget) && !aborted_warp(s_abort);
     if (here) {
       tc_fence_after();
       tmem_ld64(sb + 64 * hf, x);
@@ -313,7 +315,7 @@ __device__ __forceinline__ bool softmax_role(const AttnParams& p, const Item& it
       // O holds earlier tiles of this row: rescale this half of it once
       // O += P V of tile t-1 is done
       // (a wait that gives up marks the thread; all leave at the next tile)
-      if (!wait_all(&pv_done[(t - 1) & 1], ((t - 1) >> 1) & 1)) {
+      if (!wait_all(&pv_done[(t - 1) & 1], ((t - 1) >> 1) & 1, budget)) {
         bad = true;
       } else {
         tc_fence_after();
@@ -361,12 +363,12 @@ __device__ __forceinline__ bool softmax_role(const AttnParams& p, const Item& it
   }
   if (ok) {
     const int last = it.ntiles - 1;
-    ok = !bad && wait_all(&pv_done[last & 1], (last >> 1) & 1) && !aborted_warp(s_abort);
+    ok = !bad && wait_all(&pv_done[last & 1], (last >> 1) & 1, budget) && !aborted_warp(s_abort);
     if (ok) tc_fence_after();
   }
   if (softmax_any(!ok)) {
     if (tid == 0) {
-      set_status(p.status, ASD_ERR_TIMEOUT);
+      note_timeout(p.status);
       *s_abort = 1;
     }
     return false;
@@ -403,6 +405,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   pdl_launch_dependents();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const long long budget = wait_budget(p.status);
   Item it;
   if (!make_item(p, it)) {  // no query rows here (uniform over the CTA)
     pdl_wait();
@@ -470,9 +473,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     int chunk0 = -1;
     for (int t = 0; t < it.ntiles; ++t) {
       const int stage = t % kStages;
-      if (!wait_all(&s_kv_empty[stage], ((t / kStages) & 1) ^ 1u)) {
+      if (!wait_all(&s_kv_empty[stage], ((t / kStages) & 1) ^ 1u, budget)) {
         if (lane == 0) {
-          set_status(p.status, ASD_ERR_TIMEOUT);
+          note_timeout(p.status);
           s_abort = 1;
         }
         break;
@@ -498,14 +501,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0) {
       const uint32_t idesc_s = idesc_bf16(kRows, kKeys);         // S = Q K^T
       const uint32_t idesc_o = idesc_bf16(kRows, D, true);       // O += P V, V MN-major
-      bool mok = mbar_wait(smem_u32(&s_q_ready), 0);
+      bool mok = mbar_wait(smem_u32(&s_q_ready), 0, budget);
       if (mok) tc_fence_after();
       for (int t = 0; mok && t <= it.ntiles; ++t) {
         if (t < it.ntiles) {
           const int stage = t % kStages, b = t & 1;
-          mok = mbar_wait(smem_u32(&s_kv_full[stage]), (t / kStages) & 1);
+          mok = mbar_wait(smem_u32(&s_kv_full[stage]), (t / kStages) & 1, budget);
           // the S/P buffer is free once O += P V of tile t-2 is done
-          if (mok && t >= 2) mok = mbar_wait(smem_u32(&s_pv_done[b]), ((t >> 1) - 1) & 1);
+          if (mok && t >= 2) mok = mbar_wait(smem_u32(&s_pv_done[b]), ((t >> 1) - 1) & 1, budget);
           if (!mok || s_abort) break;
           tc_fence_after();
           const uint32_t kst = k_s0 + stage * G::kTileBytes;
@@ -520,7 +523,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (t >= 1) {
           // O += P_j V_j for the previous tile j, after its softmax
           const int j = t - 1, stage = j % kStages, b = j & 1;
-          mok = mbar_wait(smem_u32(&s_p_full[b]), (j >> 1) & 1);
+          mok = mbar_wait(smem_u32(&s_p_full[b]), (j >> 1) & 1, budget);
           if (!mok || s_abort) break;
           tc_fence_after();
           const uint32_t vst = v_s0 + stage * G::kTileBytes;
@@ -534,7 +537,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
       if (!mok) {
-        set_status(p.status, ASD_ERR_TIMEOUT);
+        note_timeout(p.status);
         s_abort = 1;
       }
       // every MMA issued above has finished before TMEM or the buffers are reused
@@ -544,7 +547,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncwarp();
   } else {
     ok = softmax_role<D>(p, it, tmem, gbase, s_anc, s_mx, s_l, &s_q_ready, s_s_full, s_p_full,
-                         s_pv_done, &s_abort, inv);
+                         s_pv_done, &s_abort, budget, inv);
   }
 
   // ------------------------------------------------------------------ finish

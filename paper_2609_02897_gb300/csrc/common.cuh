@@ -31,7 +31,8 @@ struct LmPartial {
 
 // Offsets (bytes) of the workspace regions; every region is 256-byte aligned.
 struct WsLayout {
-  size_t status;       // int32[4]: [0] first device error code
+  size_t status;       // int32[4]: [0] first device error code; [1] a bounded wait gave
+                       // up; [2..3] int64 wait budget (0: the default), set for testing
   size_t seq_flags;    // int32[B]
   size_t child_start;  // int32[T]: global slot of the node's first child
   size_t child_cnt;    // int32[T]
@@ -55,6 +56,14 @@ struct WsLayout {
 
 __device__ __forceinline__ void set_status(int* status, int code) {
   atomicCAS(status, 0, code);
+}
+
+// A bounded wait gave up: ASD_ERR_TIMEOUT as the call's status (unless an
+// earlier error came first) and word 1 of the status block set, which tells
+// the later kernels of the call that results of this one are incomplete.
+__device__ __forceinline__ void note_timeout(int* status) {
+  set_status(status, ASD_ERR_TIMEOUT);
+  atomicExch(status + 1, 1);
 }
 
 // Folds one vocabulary range's LM-head statistics (max m2, sum of exp(logit -
@@ -124,17 +133,49 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
   return ok != 0;
 }
 
+// Non-blocking test of the phase with the given parity.
+__device__ __forceinline__ bool mbar_test_wait(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
 // Waits until the phase with the given parity has completed.  Gives up after
-// kWaitCycles and returns false (the caller records ASD_ERR_TIMEOUT).
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
+// `budget` SM clock cycles (kWaitCycles unless the call set another) and
+// returns false (the caller records ASD_ERR_TIMEOUT).  try_wait may suspend
+// the thread for a while by itself, so a shortened budget (a test making a
+// wait give up) polls with the non-blocking test_wait instead.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity,
+                                          long long budget = kWaitCycles) {
+  if (budget < kWaitCycles) {
+    const long long t0 = clock64();
+    while (!mbar_test_wait(bar, parity))
+      if (clock64() - t0 > budget) return false;
+    return true;
+  }
   if (mbar_try_wait(bar, parity)) return true;
   const long long t0 = clock64();
   while (true) {
 #pragma unroll 1
     for (int i = 0; i < 32; ++i)
       if (mbar_try_wait(bar, parity)) return true;
-    if (clock64() - t0 > kWaitCycles) return false;
+    if (clock64() - t0 > budget) return false;
   }
+}
+
+// The wait budget of the kernels of one call: words 2-3 of the workspace
+// status block hold it when the host set a shorter one for testing
+// (asd_debug_set_wait_cycles), zero otherwise.  Waits for copies and MMAs
+// already in flight always use the full kWaitCycles.
+__device__ __forceinline__ long long wait_budget(const int* status) {
+  const long long b = *reinterpret_cast<const volatile long long*>(status + 2);
+  return b > 0 ? b : kWaitCycles;
 }
 
 __device__ __forceinline__ uint64_t l2_policy_evict_first() {

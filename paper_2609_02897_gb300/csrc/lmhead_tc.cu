@@ -49,14 +49,17 @@ __global__ void __launch_bounds__(192, 1)
   __shared__ __align__(8) uint64_t s_empty[kLmStages];
   __shared__ __align__(8) uint64_t s_tfull[2];
   __shared__ __align__(8) uint64_t s_tempty[2];
+  __shared__ __align__(8) uint64_t s_mma_done;
   __shared__ uint32_t s_tmem;
   __shared__ volatile int s_abort;
   __shared__ int s_pack_bad;
+  __shared__ int s_issued[kLmStages];   // fills issued per stage (drained before exit)
 
   // W and the hidden states are inputs of the step, not results of earlier
   // kernels: only the epilogue (children lists, l_draft) waits for them
   pdl_launch_dependents();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const long long budget = wait_budget(p.status);
 
   // this CTA's vocabulary range, in whole groups of kLmBoxRows rows
   const int ngroups = (p.V + kLmBoxRows - 1) / kLmBoxRows;
@@ -77,11 +80,13 @@ __global__ void __launch_bounds__(192, 1)
     for (int s = 0; s < kLmStages; ++s) {
       mbar_init(smem_u32(&s_full[s]), 1);
       mbar_init(smem_u32(&s_empty[s]), 1);
+      s_issued[s] = 0;
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(smem_u32(&s_tfull[a]), 1);
       mbar_init(smem_u32(&s_tempty[a]), 4);
     }
+    mbar_init(smem_u32(&s_mma_done), 1);
     s_abort = 0;
     // a packed weight must come from asd_pack_lm_head for this vocabulary,
     // width and range count; otherwise nothing is loaded and the error recorded
@@ -127,7 +132,7 @@ __global__ void __launch_bounds__(192, 1)
         const int ng = (min(kLmTileN, ve - v0) + kLmBoxRows - 1) / kLmBoxRows;  // 32-row groups
         for (int kp = 0; kp < nkp; ++kp) {
           const uint32_t full = smem_u32(&s_full[stage]);
-          ok = __shfl_sync(0xffffffffu, mbar_wait(smem_u32(&s_empty[stage]), ph ^ 1u), 0);
+          ok = __shfl_sync(0xffffffffu, mbar_wait(smem_u32(&s_empty[stage]), ph ^ 1u, budget), 0);
           if (!ok || s_abort) {
             ok = false;
             break;
@@ -160,6 +165,7 @@ __global__ void __launch_bounds__(192, 1)
                               v0 + j * kLmBoxRows, pol_w);
               }
             }
+            ++s_issued[stage];
           }
           __syncwarp();
           if (++stage == kLmStages) {
@@ -170,9 +176,15 @@ __global__ void __launch_bounds__(192, 1)
       }
     }
     if (!ok && lane == 0) {
-      set_status(p.status, ASD_ERR_TIMEOUT);
+      note_timeout(p.status);
       s_abort = 1;
     }
+    // every fill this CTA issued has landed before the CTA may leave
+    if (lane == 0)
+      for (int s = 0; s < kLmStages; ++s)
+        if (s_issued[s] > 0)
+          mbar_wait(smem_u32(&s_full[s]), static_cast<uint32_t>((s_issued[s] - 1) & 1));
+    __syncwarp();
   } else if (warp == 1) {
     // --------------------------------------------------------------- MMA issuer
     int stage = 0;
@@ -189,7 +201,7 @@ __global__ void __launch_bounds__(192, 1)
         // block's ng groups in the packed layout
         const int b_kstride =
             p.w_packed ? ((nrows + kLmBoxRows - 1) / kLmBoxRows) * kGroupBytes : kBTile;
-        ok = __shfl_sync(0xffffffffu, mbar_wait(smem_u32(&s_tempty[acc]), aph ^ 1u), 0);
+        ok = __shfl_sync(0xffffffffu, mbar_wait(smem_u32(&s_tempty[acc]), aph ^ 1u, budget), 0);
         if (!ok || s_abort) {
           ok = false;
           break;
@@ -197,7 +209,7 @@ __global__ void __launch_bounds__(192, 1)
         tc_fence_after();
         const uint32_t d = tmem + static_cast<uint32_t>(acc * kLmTileN);
         for (int kp = 0; kp < nkp; ++kp) {
-          ok = __shfl_sync(0xffffffffu, mbar_wait(smem_u32(&s_full[stage]), ph), 0);
+          ok = __shfl_sync(0xffffffffu, mbar_wait(smem_u32(&s_full[stage]), ph, budget), 0);
           if (!ok || s_abort) {
             ok = false;
             break;
@@ -230,9 +242,15 @@ __global__ void __launch_bounds__(192, 1)
       }
     }
     if (!ok && lane == 0) {
-      set_status(p.status, ASD_ERR_TIMEOUT);
+      note_timeout(p.status);
       s_abort = 1;
     }
+    // every tcgen05 operation of this thread is done before TMEM is released
+    if (lane == 0) {
+      tc_commit(smem_u32(&s_mma_done));
+      mbar_wait(smem_u32(&s_mma_done), 0);
+    }
+    __syncwarp();
   } else {
     // ----------------------------------------------------------------- epilogue
     const int q = warp & 3;
@@ -249,7 +267,7 @@ __global__ void __launch_bounds__(192, 1)
       for (int vt = 0; vt < nvt; ++vt) {
         const int v0 = vs + vt * kLmTileN;
         const int nrows = min(kLmTileN, ve - v0);
-        ok = __shfl_sync(0xffffffffu, mbar_wait(smem_u32(&s_tfull[acc]), aph), 0);
+        ok = __shfl_sync(0xffffffffu, mbar_wait(smem_u32(&s_tfull[acc]), aph, budget), 0);
         if (!ok || s_abort) {
           ok = false;
           break;
@@ -281,7 +299,7 @@ __global__ void __launch_bounds__(192, 1)
       }
     }
     if (!ok && lane == 0) {
-      set_status(p.status, ASD_ERR_TIMEOUT);
+      note_timeout(p.status);
       s_abort = 1;
     }
   }
@@ -338,6 +356,26 @@ __device__ __forceinline__ uint32_t cta_rank_in_cluster() {
 __device__ __forceinline__ void cluster_barrier() {
   asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;"
                ::: "memory");
+}
+
+// The shared::cluster address of this CTA's shared variable at `local` in the
+// CTA of cluster rank `rank`.
+__device__ __forceinline__ uint32_t cluster_addr(uint32_t local, int rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(local), "r"(rank));
+  return r;
+}
+__device__ __forceinline__ void st_cluster_u32(uint32_t addr, uint32_t v) {
+  asm volatile("st.shared::cluster.u32 [%0], %1;" ::"r"(addr), "r"(v) : "memory");
+}
+__device__ __forceinline__ uint32_t ld_cluster_u32(uint32_t addr) {
+  uint32_t v;
+  asm volatile("ld.shared::cluster.u32 %0, [%1];" : "=r"(v) : "r"(addr) : "memory");
+  return v;
+}
+// Counts `bytes` as arrived on the barrier's current phase without a copy.
+__device__ __forceinline__ void mbar_complete_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.complete_tx.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
 }
 
 // Bulk copy global -> shared of every CTA in `mask` (same offset, each CTA's
@@ -397,9 +435,11 @@ __global__ void __launch_bounds__(kWideThreads, 1)
   __shared__ uint32_t s_tmem;
   __shared__ volatile int s_abort;
   __shared__ int s_pack_bad;
+  __shared__ int s_issued[kWideStages];   // fills issued per stage (drained before exit)
 
   pdl_launch_dependents();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const long long budget = wait_budget(p.status);
   const int rank = CL == 2 ? static_cast<int>(cta_rank_in_cluster()) : 0;
   const uint16_t both = static_cast<uint16_t>((1u << CL) - 1u);
   // hidden rows of this launch: T, or (one level of the lazy schedule) the
@@ -432,6 +472,7 @@ __global__ void __launch_bounds__(kWideThreads, 1)
     for (int s = 0; s < kWideStages; ++s) {
       mbar_init(smem_u32(&s_full[s]), 1);
       mbar_init(smem_u32(&s_empty[s]), CL);      // every CTA of the cluster reads the stage
+      s_issued[s] = 0;
     }
     for (int a = 0; a < kWideG; ++a) {
       mbar_init(smem_u32(&s_tfull[a]), 1);
@@ -461,6 +502,13 @@ __global__ void __launch_bounds__(kWideThreads, 1)
   // 256-row vocabulary tiles (pairs of packed tiles); none when a packed
   // weight does not match (both CTAs of a cluster read the same header)
   const int nvt = s_pack_bad ? 0 : (voc.ntiles + 1) / 2;
+  // a wait that gives up stops this CTA and its peer
+  auto abort_cta = [&]() {
+    note_timeout(p.status);
+    s_abort = 1;
+    if (CL == 2)
+      st_cluster_u32(cluster_addr(smem_u32(const_cast<int*>(&s_abort)), rank ^ 1), 1u);
+  };
 
   if (warp == 0) {
     // ------------------------------------------------------------ TMA producer
@@ -494,7 +542,7 @@ __global__ void __launch_bounds__(kWideThreads, 1)
         }
         for (int kb = 0; kb < nkb; ++kb) {
           const uint32_t full = smem_u32(&s_full[stage]);
-          ok = __shfl_sync(0xffffffffu, mbar_wait(smem_u32(&s_empty[stage]), ph ^ 1u), 0);
+          ok = __shfl_sync(0xffffffffu, mbar_wait(smem_u32(&s_empty[stage]), ph ^ 1u, budget), 0);
           if (!ok || s_abort) {
             ok = false;
             break;
@@ -543,6 +591,7 @@ __global__ void __launch_bounds__(kWideThreads, 1)
                 }
               }
             }
+            ++s_issued[stage];
           }
           __syncwarp();
           if (++stage == kWideStages) {
@@ -552,10 +601,7 @@ __global__ void __launch_bounds__(kWideThreads, 1)
         }
       }
     }
-    if (!ok && lane == 0) {
-      set_status(p.status, ASD_ERR_TIMEOUT);
-      s_abort = 1;
-    }
+    if (!ok && lane == 0) abort_cta();
   } else if (warp == 1) {
     // --------------------------------------------------------------- MMA issuer
     // Accumulator use u (counted over the kernel) goes to TMEM buffer u % 2;
@@ -575,7 +621,7 @@ __global__ void __launch_bounds__(kWideThreads, 1)
         const int ncols = rows_hi > 0 ? kLmTileN + rows_hi : rows_lo;
         const uint32_t idesc = idesc_bf16(kM, (ncols + 15) & ~15);
         for (int kb = 0; kb < nkb && ok; ++kb) {
-          ok = __shfl_sync(0xffffffffu, mbar_wait(smem_u32(&s_full[stage]), ph), 0);
+          ok = __shfl_sync(0xffffffffu, mbar_wait(smem_u32(&s_full[stage]), ph, budget), 0);
           if (!ok || s_abort) {
             ok = false;
             break;
@@ -590,7 +636,8 @@ __global__ void __launch_bounds__(kWideThreads, 1)
               // the epilogue must have drained this buffer's previous tile
               ok = __shfl_sync(
                   0xffffffffu,
-                  mbar_wait(smem_u32(&s_tempty[acc]), ((static_cast<uint32_t>(u / kWideG)) & 1u) ^ 1u),
+                  mbar_wait(smem_u32(&s_tempty[acc]), ((static_cast<uint32_t>(u / kWideG)) & 1u) ^ 1u,
+                            budget),
                   0);
               if (!ok || s_abort) {
                 ok = false;
@@ -625,10 +672,7 @@ __global__ void __launch_bounds__(kWideThreads, 1)
         used += gn;
       }
     }
-    if (!ok && lane == 0) {
-      set_status(p.status, ASD_ERR_TIMEOUT);
-      s_abort = 1;
-    }
+    if (!ok && lane == 0) abort_cta();
     // every tcgen05 operation of this thread, the commits included, is done
     // before the CTA leaves the cluster
     if (lane == 0) {
@@ -664,7 +708,8 @@ __global__ void __launch_bounds__(kWideThreads, 1)
           const int u = used + g;
           const int acc = u % kWideG;
           ok = __shfl_sync(0xffffffffu,
-                           mbar_wait(smem_u32(&s_tfull[acc]), (static_cast<uint32_t>(u / kWideG)) & 1u),
+                           mbar_wait(smem_u32(&s_tfull[acc]), (static_cast<uint32_t>(u / kWideG)) & 1u,
+                                     budget),
                            0);
           if (!ok || s_abort) {
             ok = false;
@@ -717,14 +762,51 @@ __global__ void __launch_bounds__(kWideThreads, 1)
         }
       }
     }
-    if (!ok && lane == 0) {
-      set_status(p.status, ASD_ERR_TIMEOUT);
-      s_abort = 1;
-    }
+    if (!ok && lane == 0) abort_cta();
   }
 
   tc_fence_before();
   __syncthreads();
+  // From here on neither producer of the cluster issues a copy.  Every copy
+  // that lands in this CTA's shared memory (its own and, with CL = 2, the
+  // peer's half of W) has landed before the CTA leaves: the producer waits
+  // for the last phase of every stage.  The producers of a cluster are at
+  // most one phase of a stage apart (a fill needs both CTAs' MMAs to have
+  // read the previous one), so a phase that only one of them filled is either
+  // armed here for the peer's bytes or has the missing peer bytes completed
+  // here, and then waited for like the others.
+  if (CL == 2) cluster_barrier();
+  if (warp == 0 && lane == 0) {
+    for (int s = 0; s < kWideStages; ++s) {
+      const uint32_t full = smem_u32(&s_full[s]);
+      const int mine = s_issued[s];
+      const int peer =
+          CL == 2 ? static_cast<int>(ld_cluster_u32(cluster_addr(smem_u32(&s_issued[s]), rank ^ 1)))
+                  : mine;
+      // bytes of the peer's half of W in fill f of stage s (stage sequence n)
+      auto peer_bytes = [&](int f) -> uint32_t {
+        const int n = f * kWideStages + s;
+        const int vt = (n / nkb) % max(nvt, 1);
+        const int t = 2 * vt + (rank ^ 1);
+        if (CL != 2 || t >= voc.ntiles) return 0u;
+        int q, g0, ng, v0, rows;
+        voc.tile(t, p.V, q, g0, ng, v0, rows);
+        return static_cast<uint32_t>(ng * kGroupBytes);
+      };
+      if (peer == mine + 1) {
+        if (mine > 0) mbar_wait(full, static_cast<uint32_t>((mine - 1) & 1));
+        mbar_expect_tx(full, peer_bytes(mine));
+        mbar_wait(full, static_cast<uint32_t>(mine & 1));
+      } else if (mine == peer + 1) {
+        if (mine > 1) mbar_wait(full, static_cast<uint32_t>((mine - 2) & 1));
+        mbar_complete_tx(full, peer_bytes(mine - 1));
+        mbar_wait(full, static_cast<uint32_t>((mine - 1) & 1));
+      } else if (mine > 0) {
+        mbar_wait(full, static_cast<uint32_t>((mine - 1) & 1));
+      }
+    }
+  }
+  if (CL == 2) cluster_barrier();   // the peer's copies into this CTA have landed as well
   tc_fence_after();
   if (warp == 1) tmem_dealloc(tmem, kWideTmemCols);
   if (CL == 2) cluster_barrier();   // no multicast or remote arrive targets a CTA that left

@@ -98,13 +98,16 @@ __global__ void __launch_bounds__(kTailThreads) tail_kernel(const TailParams p) 
   }
 
   pdl_wait();  // every earlier kernel of the call has completed
+  // a bounded wait of an earlier kernel gave up: its statistics or verdicts
+  // are incomplete, so no sequence commits anything
+  const bool timed_out = reinterpret_cast<const volatile int*>(p.status)[1] != 0;
   const int flags = p.seq_flags ? p.seq_flags[b] : 0;
   // the drafted token's logit, loaded alongside the partials below
   const float l_draft_i =
       ((p.mode & kTailFinalize) && !tree_bad && i > 0 && i < n) ? p.l_draft[s + i] : 0.f;
   if (i == 0) {
     if (tree_bad) set_status(p.status, ASD_ERR_TREE);
-    s_skip = (tree_bad || flags) ? 1 : 0;
+    s_skip = (tree_bad || flags || timed_out) ? 1 : 0;
   }
 
   // ---------------------------------------------------------------- finalize

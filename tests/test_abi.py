@@ -24,7 +24,7 @@ def _declared():
 
 def test_every_declared_function_is_exported(lib):
     names = _declared()
-    assert len(names) == 16, names
+    assert len(names) == 17, names
     for n in names:
         assert hasattr(lib, n), n
 
@@ -218,3 +218,12 @@ def test_binding_structs_and_constants_match_header():
     assert int(defines["ASD_ABI_VERSION"]) == asd.abi_version()
     m = re.search(r"#define ASD_NOALLOC_SCRATCH_BYTES \((\d+)u << (\d+)\)", src)
     assert m and int(m.group(1)) << int(m.group(2)) == asd.NOALLOC_SCRATCH_BYTES
+
+
+def test_wait_budget_hook_checks_its_argument(lib):
+    """The failure-path test hook takes a cycle count (0: the default) and
+    refuses a negative one; it touches no GPU."""
+    lib.asd_debug_set_wait_cycles.restype = ctypes.c_int
+    lib.asd_debug_set_wait_cycles.argtypes = [ctypes.c_int64]
+    assert lib.asd_debug_set_wait_cycles(-1) == 1
+    assert lib.asd_debug_set_wait_cycles(0) == 0

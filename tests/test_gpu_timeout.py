@@ -1,0 +1,53 @@
+"""The failure path of the bounded waits (a wait that gives up), in the form
+that leaves the GPU usable: the test shortens the wait bound through the
+library's test hook (asd_debug_set_wait_cycles) so that a kernel's first
+wait on its own copy or MMA gives up, and checks that the call reports
+ASD_ERR_TIMEOUT, commits nothing (every path empty, the cache untouched,
+ctx_len_out = ctx_len), and that the next call with the default bound is
+clean and gives the results of an ordinary call bit for bit.  Covered: the
+weight-streaming LM head with the bf16 attention beside it (60-node tree) and
+the wide LM head in its unclustered form with the tensor-core attention
+(768 nodes); the clustered form of the wide LM head is not driven into a
+timeout here.  All calls go through the C ABI."""
+import numpy as np
+import pytest
+
+import _helpers as H
+
+pytestmark = pytest.mark.gpu
+
+ASD_ERR_TIMEOUT = 8
+
+
+@pytest.fixture(scope="module")
+def dev():
+    import torch
+    assert torch.cuda.is_available(), "GPU tests need a CUDA device"
+    import _device
+    return _device
+
+
+@pytest.mark.parametrize("cfg,tau", [(2, 0.3), (5, 0.3)])
+def test_a_wait_that_gives_up_reports_and_commits_nothing(dev, cfg, tau):
+    from paper_2609_02897_gb300 import asd
+    wl = H.prepared(cfg, small=True)
+    if cfg == 5:
+        # at most three 256-node pairs of tiles: the wide LM head runs unclustered
+        assert wl.T <= 768, wl.T
+    ref, status, _, _ = dev.run_verify(wl, tau)
+    assert status == 0
+    asd.asd_debug_set_wait_cycles(64)
+    try:
+        out, status, _, _ = dev.run_verify(wl, tau)
+    finally:
+        asd.asd_debug_set_wait_cycles(0)
+    assert status == ASD_ERR_TIMEOUT, asd.STATUS.get(status, status)
+    assert np.all(out["path_len"] == 0)
+    np.testing.assert_array_equal(out["ctx_len_out"], wl.ctx_len)
+    H.untouched_cache_equal(wl, out, [])
+    again, status, _, _ = dev.run_verify(wl, tau)
+    assert status == 0
+    for k in ref:
+        np.testing.assert_array_equal(again[k], ref[k], err_msg=k)
+    H.compare_verify(wl, tau, again)
+
