@@ -623,11 +623,11 @@ def roofline_of(wl, lm_ms, lm_rows, lm_passes, peak, peak_kind, tpk, tpk_kind, k
             "traffic": traffic}
 
 
-def lm_kernel_name(wl):
-    if wl.dtype != "bf16":
-        return "lmhead_f32_kernel"
-    # up to one 128-node tile: the weight-streaming kernel; more: the wide one
-    return "lmhead_tc_kernel" if wl.T <= 128 else "lmhead_wide_kernel"
+def lm_kernel_name(step):
+    """The LM-head kernel the library runs for this step (its own answer)."""
+    from paper_2609_02897_gb300 import asd
+    v = asd.asd_lm_head_variant(step.dims, step.T, step._keep[4])
+    return asd.LM_HEAD_VARIANTS.get(v, f"variant {v}")
 
 
 def workloads_block(device, stream, steps=10, warmup=3):
@@ -669,7 +669,7 @@ def workloads_block(device, stream, steps=10, warmup=3):
                            "t_bytes_us": 1e6 * t_bytes, "t_flops_us": 1e6 * t_flops},
             "stages_us": {name: 1e3 * stage_ms[j] for j, name in enumerate(STAGES)},
             "roofline": roofline_of(wl, lm_ms, wl.T, 1, peak, peak_kind, tpk, tpk_kind,
-                                    lm_kernel_name(wl), lmhead_traffic(cfg)),
+                                    lm_kernel_name(step), lmhead_traffic(cfg)),
             "mean_path_len": mean_path, "parity": par, "setup_s": t_gen,
         }
         del step, out
@@ -766,7 +766,7 @@ def run_asd(args):
     sb = step_bytes(wl, mean_path, lmb)
     fl = step_flops(wl, lm_rows)
     t_bytes, t_flops = sb / (peak * 1e9), fl / (tpk * 1e12)
-    lm_kernel = lm_kernel_name(wl)
+    lm_kernel = lm_kernel_name(step)
     if lazy:
         lm_kernel = (f"lmhead_wide_kernel + lazy_level_kernel, {lm_passes} non-empty levels of "
                      f"{wl.max_path} (LM-head stage total)")

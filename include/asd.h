@@ -299,6 +299,19 @@ const char* asd_status_string(int32_t status);
 int32_t asd_abi_version(void);
 
 /*
+ * Which LM-head kernel a call with these dims, node count and weight pointer
+ * runs (a diagnostic query; no counterpart in the paper; nothing is
+ * launched): 1 the weight-streaming tensor-core kernel (up to 128 nodes),
+ * 2 the wide kernel (more nodes, or a level of the lazy schedule), 3 the wide
+ * kernel in clusters of two SMs that multicast W between them (more than
+ * three pairs of 128-node tiles and an even range count), 4 the fp32 kernel,
+ * 0 for invalid arguments.  The clustered form multicasts from the calling
+ * GPU's own memory only: when w_lm is not device memory of the current device
+ * the call runs form 2.
+ */
+int32_t asd_lm_head_variant(const asd_dims* dims, int32_t total_nodes, const void* w_lm);
+
+/*
  * Test hook for the failure path (no counterpart in the paper).  Every wait
  * of a kernel on its own pipeline (a TMA copy, an MMA, another warp) gives up
  * after a bounded number of SM clock cycles, records ASD_ERR_TIMEOUT in the

@@ -298,9 +298,23 @@ asd_status run_attention(const Ctx& c, const void* q, const void* k_cache, const
   return err == cudaSuccess ? ASD_OK : ASD_ERR_CUDA;
 }
 
+// True when `w` is device memory of the current device (the only memory the
+// clustered LM head may multicast from).
+bool on_this_device(const void* w) {
+  int dev = 0;
+  cudaPointerAttributes a{};
+  if (cudaGetDevice(&dev) != cudaSuccess) return false;
+  if (cudaPointerGetAttributes(&a, w) != cudaSuccess) {
+    cudaGetLastError();   // an unregistered host pointer: clear the sticky-free error
+    return false;
+  }
+  return a.type == cudaMemoryTypeDevice && a.device == dev;
+}
+
 asd_status run_lmhead(const Ctx& c, const void* hidden, const void* w, float* l_draft) {
   const asd_dims& d = c.d;
   LmParams p{};
+  p.w_local = on_this_device(w) ? 1 : 0;
   p.hidden = hidden;
   p.w = w;
   p.child_start = ws_at<int32_t>(c.ws, c.L.child_start);
@@ -353,6 +367,7 @@ asd_status run_lmhead_lazy(const Ctx& c, const void* hidden, const void* w,
 
   LmParams p{};
   p.w = w;
+  p.w_local = on_this_device(w) ? 1 : 0;
   p.child_start = ws_at<int32_t>(c.ws, c.L.child_start);
   p.child_cnt = ws_at<int32_t>(c.ws, c.L.child_cnt);
   p.child_tok = ws_at<int32_t>(c.ws, c.L.child_tok);
@@ -451,6 +466,20 @@ void record(void* ev, cudaStream_t st) {
 extern "C" {
 
 int32_t asd_abi_version(void) { return ASD_ABI_VERSION; }
+
+int32_t asd_lm_head_variant(const asd_dims* dims, int32_t total_nodes, const void* w_lm) {
+  if (!dims_ok(dims) || !nodes_ok(dims, total_nodes) || !w_lm) return 0;
+  if (dims->dtype != ASD_BF16) return 4;
+  const int nsm = device_sm_count();
+  if (nsm <= 0) return 0;
+  LmParams p{};
+  p.T = total_nodes;
+  p.g_lm = lm_ranges(dims->vocab, nsm);
+  p.w_local = on_this_device(w_lm) ? 1 : 0;
+  p.t_dev = nullptr;
+  if (dims->lm_head_schedule == ASD_LM_LAZY_LEVELS) return 2;   // one level per launch
+  return lmhead_bf16_variant(p);
+}
 
 asd_status asd_debug_set_wait_cycles(int64_t cycles) {
   if (cycles < 0) return ASD_ERR_INVALID_ARG;

@@ -118,6 +118,9 @@ struct LmParams {
   // belongs to node row_node[r].  Both null: T rows, row r = node r.
   const int* t_dev;
   const int32_t* row_node;
+  // 1: W is memory of the launching device, so the wide kernel may run in
+  // clusters of two that multicast W between their SMs (set by the host)
+  int w_local;
 };
 constexpr int kLmStages = 3;       // 3 x 48 KB (a_rows <= 64): room for an attention CTA
 constexpr int kLmTileN = 128;      // vocabulary rows per MMA tile
@@ -131,6 +134,9 @@ struct LmMaps {
 };
 // bf16 path: tcgen05/TMEM GEMM with the fused max/argmax/sum-exp/l_draft epilogue.
 cudaError_t launch_lmhead_bf16(const LmParams& p, const LmMaps& maps, cudaStream_t s);
+// Which bf16 LM-head kernel launch_lmhead_bf16 runs for these parameters
+// (asd_lm_head_variant values: 1 weight-streaming, 2 wide, 3 wide in clusters).
+int lmhead_bf16_variant(const LmParams& p);
 
 // Vocabulary ranges of the LM head: range c of g covers the 32-row groups
 // [c * ngroups / g, (c + 1) * ngroups / g); each range is cut into tiles of

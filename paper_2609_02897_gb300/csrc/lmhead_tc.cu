@@ -897,18 +897,25 @@ cudaError_t launch_wide(const LmParams& p, const LmMaps& maps, cudaStream_t s) {
 }
 }  // namespace
 
+int lmhead_bf16_variant(const LmParams& p) {
+  if (p.T <= kM && !p.t_dev) return 1;
+  // several node tiles, or a row count known on the device only: the wide
+  // kernel (full 128-row node boxes).  Clusters of two pay when every CTA has
+  // at least two rounds of node pairs (the CTAs of a cluster move in lock
+  // step; with one round the coupling costs more than the halved W traffic
+  // saves), and when the ranges pair up.  Their W multicast reads this GPU's
+  // own memory only: a weight elsewhere (host or another device) runs
+  // unclustered.
+  const int pairs = (p.T + kWideG * kM - 1) / (kWideG * kM);
+  return (p.g_lm % 2 == 0 && !p.t_dev && pairs >= 4 && p.w_local) ? 3 : 2;
+}
+
 cudaError_t launch_lmhead_bf16(const LmParams& p, const LmMaps& maps, cudaStream_t s) {
   if (p.a_rows < 8 || p.a_rows > kM || p.a_rows % 8) return cudaErrorInvalidValue;
-  if (p.T > kM || p.t_dev) {
-    // several node tiles, or a row count known on the device only: the wide
-    // kernel (full 128-row node boxes).  Clusters of two pay when every CTA has
-    // at least two rounds of node pairs (the CTAs of a cluster move in lock
-    // step; with one round the coupling costs more than the halved W traffic
-    // saves), and when the ranges pair up
+  const int variant = lmhead_bf16_variant(p);
+  if (variant != 1) {
     if (p.a_rows != kM) return cudaErrorInvalidValue;
-    const int pairs = (p.T + kWideG * kM - 1) / (kWideG * kM);
-    const bool cluster = p.g_lm % 2 == 0 && !p.t_dev && pairs >= 4;
-    return cluster ? launch_wide<2>(p, maps, s) : launch_wide<1>(p, maps, s);
+    return variant == 3 ? launch_wide<2>(p, maps, s) : launch_wide<1>(p, maps, s);
   }
   const size_t smem = lmhead_tc_smem_bytes(p.a_rows);
   cudaError_t err = set_smem_attrs(lmhead_tc_kernel, smem);
