@@ -85,6 +85,9 @@ def parse():
                          "the accepted-path walk can reach")
     ap.add_argument("--no-workloads", action="store_true",
                     help="skip the tensor-bound workloads timed after the headline")
+    ap.add_argument("--batch", type=int, default=None,
+                    help="draw the workload with B sequences (a smaller case of the same shapes, "
+                         "e.g. for a profiler capture)")
     ap.add_argument("--oracle-one-step", default=None, help=argparse.SUPPRESS)
     return ap.parse_args()
 
@@ -693,7 +696,8 @@ def run_asd(args):
     if world > 1:
         dist.init_process_group("nccl", device_id=torch.device(device))
 
-    wl = synth.make_workload(CONFIG, rep=rank)
+    wl = synth.make_workload(CONFIG, rep=rank,
+                             overrides=dict(B=args.batch) if args.batch else None)
     synth.attach_tokens(wl, ranks_torch(wl, device))
     torch.cuda.empty_cache()
     is_bf16 = wl.dtype == "bf16"
@@ -828,8 +832,9 @@ def main():
     if args.oracle_one_step:
         oracle_one_step(args.oracle_one_step, args.config, args.tau)
         return
-    if args.config != CONFIG:
+    if args.config != CONFIG or args.batch:
         args.no_cpu_baseline = True   # the oracle's full step is far too slow beyond the headline
+        args.no_workloads = True
     if int(os.environ.get("WORLD_SIZE", "1")) > 1 and args.config != CONFIG:
         # replicas on several GPUs run the headline workload only: the wide LM
         # head's clustered form (steps of more than 768 nodes) serves 1-GPU runs
