@@ -312,6 +312,16 @@ int32_t asd_abi_version(void);
 int32_t asd_lm_head_variant(const asd_dims* dims, int32_t total_nodes, const void* w_lm);
 
 /*
+ * Which tree-attention kernel a call with these dims and node count runs (a
+ * diagnostic query; no counterpart in the paper; nothing is launched): 1 the
+ * bf16 split-KV kernel beside the LM head (up to 128 nodes), 2 the tensor-core
+ * kernel with one 128-row query tile per CTA, 3 the tensor-core kernel with two
+ * query tiles per CTA in ping-pong (when its 256-row items fill at least two
+ * waves of CTAs), 4 the fp32 kernel, 0 for invalid arguments.
+ */
+int32_t asd_attention_variant(const asd_dims* dims, int32_t total_nodes);
+
+/*
  * Test hook for the failure path (no counterpart in the paper).  Every wait
  * of a kernel on its own pipeline (a TMA copy, an MMA, another warp) gives up
  * after a bounded number of SM clock cycles, records ASD_ERR_TIMEOUT in the

@@ -34,7 +34,7 @@ EXPORTS = ["asd_workspace_bytes", "asd_tree_attention", "asd_lmhead_margin", "as
            "asd_abi_version", "asd_lmhead_margin_noalloc", "asd_lm_head_packed_bytes",
            "asd_pack_lm_head",
            "asd_policy_triplets", "asd_policy_init", "asd_policy_update", "asd_policy_select",
-           "asd_debug_set_wait_cycles", "asd_lm_head_variant"]
+           "asd_debug_set_wait_cycles", "asd_lm_head_variant", "asd_attention_variant"]
 
 
 class AsdError(RuntimeError):
@@ -109,6 +109,8 @@ _lib.asd_verify_step.argtypes = [_P, ctypes.POINTER(VerifyArgs), _vp, ctypes.c_s
 _lib.asd_lmhead_margin_noalloc.restype = ctypes.c_int
 _lib.asd_lmhead_margin_noalloc.argtypes = [_P] + [_vp] * 5 + [ctypes.c_int32, ctypes.c_float] + [
     _vp] * 6 + [_vp, _vp]
+_lib.asd_attention_variant.restype = ctypes.c_int32
+_lib.asd_attention_variant.argtypes = [_P, ctypes.c_int32]
 _lib.asd_lm_head_variant.restype = ctypes.c_int32
 _lib.asd_lm_head_variant.argtypes = [_P, ctypes.c_int32, _vp]
 _lib.asd_debug_set_wait_cycles.restype = ctypes.c_int
@@ -261,6 +263,16 @@ def asd_lm_head_variant(dims: Dims, total_nodes: int, w_lm) -> int:
     arguments.  `w_lm`: a tensor (device or host) or a raw address."""
     ptr = ctypes.c_void_p(w_lm.data_ptr() if hasattr(w_lm, "data_ptr") else int(w_lm))
     return int(_lib.asd_lm_head_variant(ctypes.byref(dims), int(total_nodes), ptr))
+
+
+ATTENTION_VARIANTS = {1: "attn_bf16_kernel", 2: "attn_tc_kernel", 3: "attn_pp_kernel",
+                      4: "attn_f32_kernel"}
+
+
+def asd_attention_variant(dims: Dims, total_nodes: int) -> int:
+    """Which tree-attention kernel a call runs (include/asd.h): 1-4, 0 for
+    invalid arguments."""
+    return int(_lib.asd_attention_variant(ctypes.byref(dims), int(total_nodes)))
 
 
 def asd_debug_set_wait_cycles(cycles: int):

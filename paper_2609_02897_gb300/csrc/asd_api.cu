@@ -136,6 +136,7 @@ WsLayout layout(const asd_dims& d, int T, int nsm) {
   // more than one 128-node tile: the LM head (wide kernel) leaves no room on
   // its SMs, attention runs after it on the tensor-core kernel, unsplit
   L.attn_tc = (d.dtype == ASD_BF16 && T > kAttnTcRows) ? 1 : 0;
+  if (L.attn_tc && attention_pingpong(d.batch, d.num_kv_heads, G, T, nsm)) L.attn_tc = 2;
   if (L.attn_tc) {
     L.n_splits = L.n_parts = 1;
     L.split_len = std::max(d.ctx_max, 1);
@@ -275,7 +276,7 @@ asd_status run_attention(const Ctx& c, const void* q, const void* k_cache, const
         !make_tree_tmap_bf16(&ttk, tree_k, d.head_dim, d.num_kv_heads, c.T, kAttnTcKeys) ||
         !make_tree_tmap_bf16(&ttv, tree_v, d.head_dim, d.num_kv_heads, c.T, kAttnTcKeys))
       return ASD_ERR_CUDA;
-    err = launch_attention_tc(a, tk, tv, ttk, ttv, c.st);
+    err = launch_attention_tc(a, tk, tv, ttk, ttv, c.L.attn_tc == 2, c.st);
   } else if (d.dtype == ASD_BF16) {
     CUtensorMap tk, tv;
     uint64_t rows;
@@ -466,6 +467,15 @@ void record(void* ev, cudaStream_t st) {
 extern "C" {
 
 int32_t asd_abi_version(void) { return ASD_ABI_VERSION; }
+
+int32_t asd_attention_variant(const asd_dims* dims, int32_t total_nodes) {
+  if (!dims_ok(dims) || !nodes_ok(dims, total_nodes)) return 0;
+  if (dims->dtype != ASD_BF16) return 4;
+  const int nsm = device_sm_count();
+  if (nsm <= 0) return 0;
+  const WsLayout L = layout(*dims, total_nodes, nsm);
+  return L.attn_tc == 2 ? 3 : (L.attn_tc == 1 ? 2 : 1);
+}
 
 int32_t asd_lm_head_variant(const asd_dims* dims, int32_t total_nodes, const void* w_lm) {
   if (!dims_ok(dims) || !nodes_ok(dims, total_nodes) || !w_lm) return 0;

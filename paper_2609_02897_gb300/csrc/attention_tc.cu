@@ -591,27 +591,530 @@ __global__ void __launch_bounds__(kThreads, 1)
   pdl_wait();   // the next kernel's wait covers every earlier kernel
 }
 
+// ----------------------------------------------------------------------------
+// Ping-pong variant: one CTA per (256 query rows, sequence x KV head) = two
+// 128-row query tiles A and B that see the same keys.  Every K/V tile serves
+// both: S_A = Q_A.K^T and S_B = Q_B.K^T, then O_A += P_A.V and O_B += P_B.V, so
+// the MMAs of one tile run while the other tile's softmax works, and a K/V
+// byte feeds twice the products.  Q stays in shared memory (both tiles, 128-byte
+// swizzled, written by the softmax threads); TMEM holds O_A [0, D),
+// O_B [D, 2D) and S/P_A [256, 384), S/P_B [384, 512).  K and V come through
+// separate rings with their own barriers, so a K slot is refilled as soon as
+// both S MMAs have read it.  Warps: 0 TMA producer, 1 MMA issuer (lane 0),
+// 2-5 softmax of tile A, 6-9 softmax of tile B; a softmax thread owns one row
+// of its tile and all 128 keys of every key tile, so no exchange between warps
+// is needed: per key tile it reads S twice (the row max, then the
+// exponentials) and writes P as bf16 pairs over the S columns already read.
+constexpr int kPPRows = 2 * kRows;   // query rows per CTA
+
+template <int D>
+struct PPGeom {
+  static constexpr int kNH = D / 64;
+  static constexpr int kStages = D == 64 ? 3 : 2;
+  static constexpr int kQTile = kNH * kRows * 128;    // one query tile
+  static constexpr int kKVTile = kNH * kKeys * 128;   // one K or one V tile
+  static constexpr int kQOff = 0;
+  static constexpr int kKOff = 2 * kQTile;
+  static constexpr int kVOff = kKOff + kStages * kKVTile;
+  static constexpr int kBytes = kVOff + kStages * kKVTile;
+};
+
+__device__ __forceinline__ bool make_item_pp(const AttnParams& p, Item& it) {
+  const int rb = blockIdx.x, bg = blockIdx.y;
+  it.b = bg / p.Hkv;
+  it.g = bg - it.b * p.Hkv;
+  it.s0 = p.cu_nodes[it.b];
+  it.n = p.cu_nodes[it.b + 1] - it.s0;
+  it.R = it.n * p.G;
+  it.r0 = rb * kPPRows;
+  if (it.n <= 0 || it.n > kMaxNodes || it.s0 < 0 || it.s0 + it.n > p.T || it.r0 >= it.R)
+    return false;
+  it.nrows = min(kPPRows, it.R - it.r0);
+  it.ctx = min(max(p.ctx_len[it.b], 0), p.ctx_max);
+  it.nctx = (it.ctx + kKeys - 1) / kKeys;
+  it.ntree = (it.n + kKeys - 1) / kKeys;
+  it.ntiles = it.nctx + it.ntree;
+  return true;
+}
+
+// Issues one K (which = 0) or V (which = 1) tile t into `dst` (producer lane 0;
+// contiguous cache or tree keys).
+template <int D>
+__device__ __forceinline__ void issue_half_tile(const AttnParams& p, const Item& it, int t,
+                                                uint32_t dst, uint32_t bar,
+                                                const CUtensorMap* tm, const CUtensorMap* tm_tree,
+                                                uint64_t pol) {
+  using G = PPGeom<D>;
+  mbar_expect_tx(bar, G::kKVTile);
+  if (t >= it.nctx) {
+    const int key0 = (t - it.nctx) * kKeys;
+#pragma unroll
+    for (int h = 0; h < G::kNH; ++h)
+      tma_load_3d(dst + h * (kKeys * 128), tm_tree, bar, h * 64, it.g, it.s0 + key0, pol);
+    return;
+  }
+  const int row = (it.b * p.Hkv + it.g) * p.ctx_max + t * kKeys;
+#pragma unroll
+  for (int h = 0; h < G::kNH; ++h) tma_load_2d(dst + h * (kKeys * 128), tm, bar, h * 64, row, pol);
+}
+
+// Paged context tile t, K or V (the whole producer warp; see issue_paged_tile).
+template <int D>
+__device__ __forceinline__ void issue_paged_half(const AttnParams& p, const Item& it, int t,
+                                                 uint32_t dst, uint32_t bar, const CUtensorMap* tm,
+                                                 uint64_t pol, int* s_pages, int& chunk0,
+                                                 int lane) {
+  using G = PPGeom<D>;
+  const int ps = p.page_size;
+  const int br = ps < kKeys ? ps : kKeys;
+  const int nbox = kKeys / br;
+  const int key0 = t * kKeys;
+  const int e_first = key0 / ps, e_last = (key0 + (nbox - 1) * br) / ps;
+  if (chunk0 < 0 || e_first < chunk0 || e_last >= chunk0 + kPageChunk) {
+    chunk0 = e_first;
+    const int32_t* row_pt = p.page_table + static_cast<size_t>(it.b) * p.pages_per_seq;
+    for (int i = lane; i < kPageChunk; i += 32) {
+      const int e = chunk0 + i;
+      s_pages[i] = e < p.pages_per_seq ? row_pt[e] : -1;
+    }
+    __syncwarp();
+  }
+  int row = -1;
+  if (lane < nbox) {
+    const int key = key0 + lane * br;
+    if (key < it.ctx) {
+      const int page = s_pages[key / ps - chunk0];
+      if (page < 0 || page >= p.num_pages)
+        set_status(p.status, ASD_ERR_CTX_RANGE);
+      else
+        row = (page * p.Hkv + it.g) * ps + (key % ps);
+    }
+  }
+  const uint32_t valid = __ballot_sync(0xffffffffu, row >= 0);
+  if (lane == 0) mbar_expect_tx(bar, static_cast<uint32_t>(__popc(valid) * G::kNH * br * 128));
+  __syncwarp();
+  if (row >= 0) {
+#pragma unroll
+    for (int h = 0; h < G::kNH; ++h)
+      tma_load_2d(dst + h * (kKeys * 128) + lane * br * 128, tm, bar, h * 64, row, pol);
+  }
+  __syncwarp();
+}
+
+template <int D>
+__global__ void __launch_bounds__(kThreads, 1)
+    attn_pp_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_v,
+                   const __grid_constant__ CUtensorMap tm_tk,
+                   const __grid_constant__ CUtensorMap tm_tv, const AttnParams p) {
+  using G = PPGeom<D>;
+  constexpr int S = G::kStages;
+  extern __shared__ uint8_t smem_raw[];
+  __shared__ __align__(8) uint64_t s_k_full[S], s_k_empty[S], s_v_full[S], s_v_empty[S];
+  __shared__ __align__(8) uint64_t s_s_full[2];    // S of tile X computed (MMA -> softmax X)
+  __shared__ __align__(8) uint64_t s_p_full[2];    // P of tile X written (softmax X -> MMA)
+  __shared__ __align__(8) uint64_t s_pv_done[2];   // O_X += P_X V done (MMA -> softmax X)
+  __shared__ __align__(8) uint64_t s_q_ready;
+  __shared__ __align__(8) uint64_t s_mma_done;
+  __shared__ uint32_t s_tmem;
+  __shared__ volatile int s_abort;
+  __shared__ int s_par[kMaxNodes];
+  __shared__ uint64_t s_anc[kMaxNodes][2];
+  __shared__ int s_pages[kPageChunk];
+  __shared__ int s_issued[2][S];   // producer: K (0) and V (1) fills issued per stage
+
+  pdl_launch_dependents();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const long long budget = wait_budget(p.status);
+  Item it;
+  if (!make_item_pp(p, it)) {  // no query rows here (uniform over the CTA)
+    pdl_wait();
+    return;
+  }
+  const int nx = it.nrows > kRows ? 2 : 1;   // query tiles present
+
+  uint32_t base = smem_u32(smem_raw);
+  const uint32_t pad = (1024u - (base & 1023u)) & 1023u;
+  uint8_t* gbase = smem_raw + pad;
+  base += pad;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < S; ++s) {
+      mbar_init(smem_u32(&s_k_full[s]), 1);
+      mbar_init(smem_u32(&s_k_empty[s]), 1);
+      mbar_init(smem_u32(&s_v_full[s]), 1);
+      mbar_init(smem_u32(&s_v_empty[s]), 1);
+      s_issued[0][s] = s_issued[1][s] = 0;
+    }
+    for (int x = 0; x < 2; ++x) {
+      mbar_init(smem_u32(&s_s_full[x]), 1);
+      mbar_init(smem_u32(&s_p_full[x]), 4);
+      mbar_init(smem_u32(&s_pv_done[x]), 1);
+    }
+    mbar_init(smem_u32(&s_q_ready), 8);
+    mbar_init(smem_u32(&s_mma_done), 1);
+    s_abort = 0;
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(&s_tmem), kTmemCols);
+    tmem_relinquish();
+  }
+  for (int i = threadIdx.x; i < it.n; i += kThreads) s_par[i] = p.parent[it.s0 + i];
+  __syncthreads();
+  for (int i = threadIdx.x; i < it.n; i += kThreads) {
+    uint64_t lo = 0, hi = 0;
+    int u = i;
+    while (true) {
+      if (u < 64) lo |= 1ull << u; else hi |= 1ull << (u - 64);
+      const int pu = s_par[u];
+      if (pu < 0 || pu >= u) break;
+      u = pu;
+    }
+    s_anc[i][0] = lo;
+    s_anc[i][1] = hi;
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = s_tmem;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ TMA producer
+    // K(t) then V(t), each into its own ring; K slots free up as soon as both
+    // S MMAs of their tile are done, V slots after both P.V MMAs
+    if (lane == 0) {
+      prefetch_tmap(&tm_k);
+      prefetch_tmap(&tm_v);
+      prefetch_tmap(&tm_tk);
+      prefetch_tmap(&tm_tv);
+    }
+    const uint64_t pol = l2_policy_evict_first();
+    int chunk0 = -1;
+    bool ok = true;
+    for (int t = 0; t < it.ntiles && ok; ++t) {
+      const int stage = t % S;
+      const uint32_t ph = ((t / S) & 1) ^ 1u;
+#pragma unroll
+      for (int which = 0; which < 2; ++which) {
+        uint64_t* empty = which ? &s_v_empty[stage] : &s_k_empty[stage];
+        uint64_t* full = which ? &s_v_full[stage] : &s_k_full[stage];
+        if (!wait_all(empty, ph, budget) || aborted_warp(&s_abort)) {
+          ok = false;
+          break;
+        }
+        const uint32_t dst = base + (which ? G::kVOff : G::kKOff) + stage * G::kKVTile;
+        if (p.page_size != 0 && t < it.nctx)
+          issue_paged_half<D>(p, it, t, dst, smem_u32(full), which ? &tm_v : &tm_k, pol, s_pages,
+                              chunk0, lane);
+        else if (lane == 0)
+          issue_half_tile<D>(p, it, t, dst, smem_u32(full), which ? &tm_v : &tm_k,
+                             which ? &tm_tv : &tm_tk, pol);
+        if (lane == 0) ++s_issued[which][stage];
+        __syncwarp();
+      }
+    }
+    if (!ok && lane == 0) {
+      note_timeout(p.status);
+      s_abort = 1;
+    }
+    // every copy issued has landed before the buffers are reused or left
+    if (lane == 0)
+      for (int which = 0; which < 2; ++which)
+        for (int s = 0; s < S; ++s)
+          if (s_issued[which][s] > 0)
+            mbar_wait(smem_u32(which ? &s_v_full[s] : &s_k_full[s]),
+                      static_cast<uint32_t>((s_issued[which][s] - 1) & 1));
+    __syncwarp();
+  } else if (warp == 1) {
+    // --------------------------------------------------------------- MMA issuer
+    if (lane == 0) {
+      const uint32_t idesc_s = idesc_bf16(kRows, kKeys);         // S = Q K^T
+      const uint32_t idesc_o = idesc_bf16(kRows, D, true);       // O += P V, V MN-major
+      bool mok = mbar_wait(smem_u32(&s_q_ready), 0, budget);
+      if (mok) tc_fence_after();
+      // S_x(t) = Q_x K(t)^T into tile x's S/P columns; they are free once
+      // O_x += P_x V of tile t-1 is done.  The last S of tile t releases K(t).
+      auto issue_s = [&](int x, int t) -> bool {
+        const int stage = t % S;
+        if (!mbar_wait(smem_u32(&s_k_full[stage]), (t / S) & 1, budget) || s_abort) return false;
+        if (t > 0 && (!mbar_wait(smem_u32(&s_pv_done[x]), (t - 1) & 1, budget) || s_abort))
+          return false;
+        tc_fence_after();
+        const uint32_t kst = base + G::kKOff + stage * G::kKVTile;
+        const uint32_t qst = base + G::kQOff + x * G::kQTile;
+#pragma unroll
+        for (int ks = 0; ks < D / 16; ++ks) {
+          const int h = ks >> 2, kk = ks & 3;
+          tc_mma(tmem + (256u + 128u * static_cast<uint32_t>(x)),
+                 sw128_desc(qst + h * (kRows * 128) + 32 * kk),
+                 sw128_desc(kst + h * (kKeys * 128) + 32 * kk), idesc_s, ks > 0 ? 1u : 0u);
+        }
+        tc_commit(smem_u32(&s_s_full[x]));
+        if (x == nx - 1) tc_commit(smem_u32(&s_k_empty[stage]));
+        return true;
+      };
+      // O_x += P_x(t) V(t) once tile x's softmax of tile t is done; the last
+      // P.V of tile t releases V(t)
+      auto issue_pv = [&](int x, int t) -> bool {
+        const int stage = t % S;
+        if (!mbar_wait(smem_u32(&s_v_full[stage]), (t / S) & 1, budget) || s_abort) return false;
+        if (!mbar_wait(smem_u32(&s_p_full[x]), t & 1, budget) || s_abort) return false;
+        tc_fence_after();
+        const uint32_t vst = base + G::kVOff + stage * G::kKVTile;
+#pragma unroll
+        for (int kk = 0; kk < kKeys / 16; ++kk)
+          tc_mma_ts(tmem + static_cast<uint32_t>(x * D),
+                    tmem + (256u + 128u * static_cast<uint32_t>(x)) + kk * 8,
+                    sw128_desc_mn(vst + kk * 2048, kKeys * 128, 1024), idesc_o,
+                    (t > 0 || kk > 0) ? 1u : 0u);
+        tc_commit(smem_u32(&s_pv_done[x]));
+        if (x == nx - 1) tc_commit(smem_u32(&s_v_empty[stage]));
+        return true;
+      };
+      // ping-pong: while tile A's softmax works on tile t, the tensor cores
+      // run O_B += P_B V(t-1) and S_B(t); while B's works, O_A += P_A V(t) and
+      // S_A(t+1)
+      for (int x = 0; mok && x < nx; ++x) mok = issue_s(x, 0);
+      for (int t = 0; mok && t < it.ntiles; ++t) {
+        for (int x = 0; mok && x < nx; ++x) {
+          mok = issue_pv(x, t);
+          if (mok && t + 1 < it.ntiles) mok = issue_s(x, t + 1);
+        }
+      }
+      if (!mok) {
+        note_timeout(p.status);
+        s_abort = 1;
+      }
+      // every MMA issued above has finished before TMEM or the buffers are reused
+      tc_commit(smem_u32(&s_mma_done));
+      mbar_wait(smem_u32(&s_mma_done), 0);
+    }
+    __syncwarp();
+  } else {
+    // ------------------------------------------------------------ softmax of tile x
+    const int x = (warp - 2) >> 2;
+    const int row = (warp & 3) * 32 + lane;    // = TMEM lane = row of the tile
+    const int rr = x * kRows + row;            // row of the item
+    const bool mine = rr < it.nrows;
+    const uint32_t lane_base = tmem + (static_cast<uint32_t>((warp & 3) * 32) << 16);
+    const uint32_t sb = lane_base + (256u + 128u * static_cast<uint32_t>(x));
+    // the row's query -> shared memory, 128-byte swizzled like a TMA tile
+    {
+      const int q_row = it.r0 + rr;
+      const int node = q_row / p.G;
+      const uint4* qg = reinterpret_cast<const uint4*>(
+          static_cast<const __nv_bfloat16*>(p.q) +
+          (mine ? (static_cast<size_t>(it.s0 + node) * p.Hq + it.g * p.G + (q_row - node * p.G)) : 0) *
+              D);
+      uint8_t* qs = gbase + G::kQOff + x * G::kQTile;
+#pragma unroll
+      for (int c = 0; c < D / 8; ++c) {
+        const uint4 v = mine ? qg[c] : make_uint4(0u, 0u, 0u, 0u);
+        *reinterpret_cast<uint4*>(qs + (c >> 3) * (kRows * 128) + row * 128 +
+                                  (((c & 7) ^ (row & 7)) << 4)) = v;
+      }
+      fence_proxy_async();   // the tensor cores read these rows
+      __syncwarp();
+      if (lane == 0) mbar_arrive(smem_u32(&s_q_ready));
+    }
+    uint64_t alo = 0, ahi = 0;
+    if (mine) {
+      const int node = (it.r0 + rr) / p.G;
+      alo = s_anc[node][0];
+      ahi = s_anc[node][1];
+    }
+    // a second query tile with no rows: its warps only staged the zero rows
+    if (x < nx) {
+    const float c = p.scale_log2;
+    float m_ref = -INFINITY, l = 0.f;
+    bool ok = true;
+    for (int t = 0; t < it.ntiles; ++t) {
+      const bool tree = t >= it.nctx;
+      const int key0 = tree ? (t - it.nctx) * kKeys : t * kKeys;
+      const int valid = min(kKeys, (tree ? it.n : it.ctx) - key0);
+      ok = wait_all(&s_s_full[x], t & 1, budget) && !aborted_warp(&s_abort);
+      if (!ok) break;
+      tc_fence_after();
+      // pass 1: the row's max over the tile's keys (raw scores); only a
+      // ragged context tile and the tree tile need the key mask
+      const bool masked = tree || valid < kKeys;
+      float mt = -INFINITY;
+#pragma unroll
+      for (int hf = 0; hf < 2; ++hf) {
+        float xs[64];
+        tmem_ld64(sb + 64 * hf, xs);
+        if (masked) {
+#pragma unroll
+          for (int k = 0; k < 64; ++k) {
+            const int key = 64 * hf + k;
+            bool v = key < valid;
+            if (tree) v = v && anc_bit(alo, ahi, key0 + key);
+            xs[k] = v ? xs[k] : -INFINITY;
+          }
+        }
+#pragma unroll
+        for (int k = 0; k < 64; ++k) mt = fmaxf(mt, xs[k]);
+      }
+      mt *= c;
+      const float mn = fmaxf(m_ref, mt);
+      const bool had = m_ref != -INFINITY;
+      const bool need = had ? (mn > m_ref + kRescaleLog2) : (mn != -INFINITY);
+      if (__any_sync(0xffffffffu, need && had)) {
+        // O holds earlier tiles of this row: rescale it once O += P V of tile
+        // t-1 is done
+        if (!wait_all(&s_pv_done[x], (t - 1) & 1, budget)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const float alpha = (need && had) ? exp2f(m_ref - mn) : 1.f;
+#pragma unroll 1
+        for (int cc = 0; cc < D / 32; ++cc) {
+          float o[32];
+          const uint32_t oc = lane_base + static_cast<uint32_t>(x * D) + 32 * cc;
+          tmem_ld32(oc, o);
+#pragma unroll
+          for (int i = 0; i < 32; ++i) o[i] *= alpha;
+          tmem_st32(oc, o);
+        }
+      }
+      if (need) {
+        l = had ? l * exp2f(m_ref - mn) : 0.f;
+        m_ref = mn;
+      }
+      const float mu = (m_ref == -INFINITY) ? 0.f : m_ref;
+      // pass 2: P = exp2(s c - m) as bf16 pairs over the S columns already read
+#pragma unroll
+      for (int hf = 0; hf < 2; ++hf) {
+        float xs[64];
+        tmem_ld64(sb + 64 * hf, xs);
+        if (masked) {
+#pragma unroll
+          for (int k = 0; k < 64; ++k) {
+            const int key = 64 * hf + k;
+            bool v = key < valid;
+            if (tree) v = v && anc_bit(alo, ahi, key0 + key);
+            xs[k] = v ? xs[k] : -INFINITY;
+          }
+        }
+        uint32_t pk[32];
+#pragma unroll
+        for (int k = 0; k < 64; k += 2) {
+          const float p0 = ex2_approx(fmaf(xs[k], c, -mu)), p1 = ex2_approx(fmaf(xs[k + 1], c, -mu));
+          l += p0 + p1;
+          __nv_bfloat162 h = __floats2bfloat162_rn(p0, p1);
+          pk[k / 2] = *reinterpret_cast<uint32_t*>(&h);
+        }
+        tmem_st32u(sb + 32 * hf, pk);
+      }
+      if (valid < kKeys && x == 0) {
+        // ragged tile: V rows past the last valid key may hold anything; zero
+        // them (once the tile has landed) so that 0 * V stays 0 for both tiles
+        const int stage = t % S;
+        if (!wait_all(&s_v_full[stage], (t / S) & 1, budget)) {
+          ok = false;
+          break;
+        }
+        uint8_t* vt = gbase + G::kVOff + stage * G::kKVTile;
+        constexpr int kChunksPerRow = G::kNH * 8;
+        for (int i = threadIdx.x - 64; i < (kKeys - valid) * kChunksPerRow; i += 128) {
+          const int r = valid + i / kChunksPerRow, rem = i % kChunksPerRow;
+          *reinterpret_cast<uint4*>(vt + (rem >> 3) * (kKeys * 128) + r * 128 + (rem & 7) * 16) =
+              make_uint4(0u, 0u, 0u, 0u);
+        }
+        fence_proxy_async();
+        // the four warps of tile A zero disjoint rows; each arrives for itself
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(smem_u32(&s_p_full[x]));
+    }
+    if (ok) {
+      const int last = it.ntiles - 1;
+      ok = wait_all(&s_pv_done[x], last & 1, budget) && !aborted_warp(&s_abort);
+      if (ok) tc_fence_after();
+    }
+    if (!ok) {
+      if (lane == 0) {
+        note_timeout(p.status);
+        s_abort = 1;
+      }
+    } else {
+      // O_x / l -> the row's output, D columns
+      const float inv = l > 0.f ? 1.f / l : 0.f;
+      __nv_bfloat16* out = nullptr;
+      if (mine) {
+        const int q_row = it.r0 + rr;
+        const int node = q_row / p.G;
+        out = static_cast<__nv_bfloat16*>(p.out) +
+              (static_cast<size_t>(it.s0 + node) * p.Hq + it.g * p.G + (q_row - node * p.G)) * D;
+      }
+#pragma unroll 1
+      for (int cc = 0; cc < D / 32; ++cc) {
+        float o[32];
+        tmem_ld32(lane_base + static_cast<uint32_t>(x * D) + 32 * cc, o);
+        if (mine) {
+#pragma unroll
+          for (int k = 0; k < 32; k += 8) {
+            uint4 pk;
+            __nv_bfloat162 h0 = __floats2bfloat162_rn(o[k] * inv, o[k + 1] * inv);
+            __nv_bfloat162 h1 = __floats2bfloat162_rn(o[k + 2] * inv, o[k + 3] * inv);
+            __nv_bfloat162 h2 = __floats2bfloat162_rn(o[k + 4] * inv, o[k + 5] * inv);
+            __nv_bfloat162 h3 = __floats2bfloat162_rn(o[k + 6] * inv, o[k + 7] * inv);
+            pk.x = *reinterpret_cast<uint32_t*>(&h0);
+            pk.y = *reinterpret_cast<uint32_t*>(&h1);
+            pk.z = *reinterpret_cast<uint32_t*>(&h2);
+            pk.w = *reinterpret_cast<uint32_t*>(&h3);
+            *reinterpret_cast<uint4*>(out + 32 * cc + k) = pk;
+          }
+        }
+      }
+    }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc(tmem, kTmemCols);
+  pdl_wait();   // the next kernel's wait covers every earlier kernel
+}
+
 }  // namespace
 
-size_t attention_tc_smem_bytes(int head_dim) {
+size_t attention_tc_smem_bytes(int head_dim, bool pingpong) {
+  if (pingpong)
+    return 1024 + static_cast<size_t>(head_dim == 64 ? PPGeom<64>::kBytes : PPGeom<128>::kBytes);
   return 1024 + static_cast<size_t>(head_dim == 64 ? TcGeom<64>::kBytes : TcGeom<128>::kBytes);
+}
+
+bool attention_pingpong(int batch, int num_kv_heads, int G, int total_nodes, int nsm) {
+  // the ping-pong kernel does two query tiles per CTA: it pays once its items
+  // fill at least two waves of CTAs (measured: 1.2x the single-tile kernel's
+  // work per SM; with fewer items the single-tile kernel keeps more SMs busy)
+  const long long rows = static_cast<long long>(total_nodes) * G;
+  const long long items = static_cast<long long>(num_kv_heads) * ((rows + kPPRows - 1) / kPPRows);
+  return batch > 0 && items >= 2LL * nsm;
 }
 
 cudaError_t launch_attention_tc(const AttnParams& p, const CUtensorMap& tm_k,
                                 const CUtensorMap& tm_v, const CUtensorMap& tm_tk,
-                                const CUtensorMap& tm_tv, cudaStream_t s) {
-  const dim3 grid((p.max_nodes * p.G + kRows - 1) / kRows, p.B * p.Hkv, 1);
-  const size_t smem = attention_tc_smem_bytes(p.D);
+                                const CUtensorMap& tm_tv, bool pingpong, cudaStream_t s) {
+  const size_t smem = attention_tc_smem_bytes(p.D, pingpong);
+  if (p.D != 64 && p.D != 128) return cudaErrorInvalidValue;
   cudaError_t err;
-  if (p.D == 64) {
-    err = set_smem_attrs(attn_tc_kernel<64>, smem);
+  if (pingpong) {
+    const dim3 grid((p.max_nodes * p.G + kPPRows - 1) / kPPRows, p.B * p.Hkv, 1);
+    auto* k = p.D == 64 ? attn_pp_kernel<64> : attn_pp_kernel<128>;
+    err = set_smem_attrs(k, smem);
     if (err != cudaSuccess) return err;
-    return launch_pdl(attn_tc_kernel<64>, grid, dim3(kThreads), smem, s, tm_k, tm_v, tm_tk, tm_tv, p);
+    return launch_pdl(k, grid, dim3(kThreads), smem, s, tm_k, tm_v, tm_tk, tm_tv, p);
   }
-  if (p.D != 128) return cudaErrorInvalidValue;
-  err = set_smem_attrs(attn_tc_kernel<128>, smem);
+  const dim3 grid((p.max_nodes * p.G + kRows - 1) / kRows, p.B * p.Hkv, 1);
+  auto* k = p.D == 64 ? attn_tc_kernel<64> : attn_tc_kernel<128>;
+  err = set_smem_attrs(k, smem);
   if (err != cudaSuccess) return err;
-  return launch_pdl(attn_tc_kernel<128>, grid, dim3(kThreads), smem, s, tm_k, tm_v, tm_tk, tm_tv, p);
+  return launch_pdl(k, grid, dim3(kThreads), smem, s, tm_k, tm_v, tm_tk, tm_tv, p);
 }
 
 }  // namespace asd

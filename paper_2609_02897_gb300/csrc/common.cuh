@@ -49,7 +49,9 @@ struct WsLayout {
   size_t lz_rows;      // int32[2][T]: node ids of a level's rows (two levels in flight)
   size_t lz_h;         // bf16[2][lz_cap][hidden]: their hidden rows
   int lz_cap;          // T rounded up to 128
-  int attn_tc;         // 1: the tensor-core attention kernel (attention has the SMs to itself)
+  int attn_tc;         // tensor-core attention (attention has the SMs to itself): 1 one
+                       // query tile per CTA, 2 two query tiles in ping-pong; 0: the bf16
+                       // mma.sync or the fp32 kernel
 };
 
 // ---------------------------------------------------------------- device utils

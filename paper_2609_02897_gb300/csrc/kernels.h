@@ -91,12 +91,16 @@ int attention_keys_per_tile();   // context keys per K/V tile = TMA box rows
 // tm_v: 2D maps over the cache rows with boxes of 64 columns x
 // min(kAttnTcKeys, rows per page) rows; tm_tk / tm_tv: 3D maps over the tree
 // K/V [T, Hkv, D] with boxes of 64 columns x 1 head x kAttnTcKeys nodes.
-constexpr int kAttnTcRows = 128;   // query rows per CTA
+// pingpong: the two-query-tile form (256 rows per CTA: one tile's MMAs run
+// during the other's softmax), chosen by attention_pingpong() when its items
+// fill at least two waves of CTAs.
+constexpr int kAttnTcRows = 128;   // query rows per CTA (per tile of the ping-pong form)
 constexpr int kAttnTcKeys = 128;   // keys per tile
-size_t attention_tc_smem_bytes(int head_dim);
+size_t attention_tc_smem_bytes(int head_dim, bool pingpong);
+bool attention_pingpong(int batch, int num_kv_heads, int G, int total_nodes, int nsm);
 cudaError_t launch_attention_tc(const AttnParams& p, const CUtensorMap& tm_k,
                                 const CUtensorMap& tm_v, const CUtensorMap& tm_tk,
-                                const CUtensorMap& tm_tv, cudaStream_t s);
+                                const CUtensorMap& tm_tv, bool pingpong, cudaStream_t s);
 
 // -------------------------------------------------------------------- LM head
 struct LmParams {

@@ -48,3 +48,22 @@ def test_small_trees_and_fp32(dev):
     tiny = synth.make_workload(1)
     assert asd.asd_lm_head_variant(dev.dims_of(tiny), tiny.T, w_dev) == 4
     assert asd.asd_lm_head_variant(dev.dims_of(small), 0, w_dev) == 0
+
+
+def test_attention_variant(dev):
+    import torch
+    from paper_2609_02897_gb300 import asd
+    nsm = torch.cuda.get_device_properties(0).multi_processor_count
+    small = synth.make_workload(2, small=True)
+    assert asd.asd_attention_variant(dev.dims_of(small), small.T) == 1
+    tiny = synth.make_workload(1)
+    assert asd.asd_attention_variant(dev.dims_of(tiny), tiny.T) == 4
+    wl = synth.make_workload(5, small=True)        # 6 x 128 nodes, 2 KV heads, G = 4
+    dims = dev.dims_of(wl)
+    assert asd.asd_attention_variant(dims, wl.T) == 2
+    # the two-tile form once its 256-row items fill two waves of CTAs
+    dims.batch = 4 * nsm
+    items = dims.num_kv_heads * ((dims.batch * 128 * 4 + 255) // 256)
+    assert items >= 2 * nsm
+    assert asd.asd_attention_variant(dims, dims.batch * 128) == 3
+    assert asd.asd_attention_variant(dims, 0) == 0
