@@ -58,10 +58,6 @@ struct TcGeom {
   static constexpr int kBytes = kVOff + kStages * kTileBytes;
 };
 
-__device__ __forceinline__ bool anc_bit(uint64_t lo, uint64_t hi, int j) {
-  return j < 64 ? ((lo >> j) & 1ull) : ((hi >> (j - 64)) & 1ull);
-}
-
 // Named barrier 1 of the eight softmax warps.
 __device__ __forceinline__ void softmax_sync() {
   asm volatile("bar.sync 1, %0;" ::"n"(kSoftmaxThreads) : "memory");
@@ -290,11 +286,12 @@ __device__ __forceinline__ bool softmax_role(const AttnParams& p, const Item& it
       tc_fence_after();
       tmem_ld64(sb + 64 * hf, x);
       if (tree || valid < kKeys) {
+        // the tree tile holds every node of the sequence (at most 128) from
+        // key 0: key k of this half is bit k of the half's ancestor word
+        const uint64_t am = tree ? (hf ? ahi : alo) : ~0ull;
 #pragma unroll
         for (int k = 0; k < 64; ++k) {
-          const int key = 64 * hf + k;
-          bool v = key < valid;
-          if (tree) v = v && anc_bit(alo, ahi, key0 + key);
+          const bool v = (64 * hf + k < valid) && ((am >> k) & 1ull);
           x[k] = v ? x[k] : -INFINITY;
         }
       }
@@ -944,11 +941,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         float xs[64];
         tmem_ld64(sb + 64 * hf, xs);
         if (masked) {
+          // the tree tile holds every node of the sequence (at most 128) from
+          // key 0: key k of this half is bit k of the half's ancestor word
+          const uint64_t am = tree ? (hf ? ahi : alo) : ~0ull;
 #pragma unroll
           for (int k = 0; k < 64; ++k) {
-            const int key = 64 * hf + k;
-            bool v = key < valid;
-            if (tree) v = v && anc_bit(alo, ahi, key0 + key);
+            const bool v = (64 * hf + k < valid) && ((am >> k) & 1ull);
             xs[k] = v ? xs[k] : -INFINITY;
           }
         }
@@ -989,11 +987,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         float xs[64];
         tmem_ld64(sb + 64 * hf, xs);
         if (masked) {
+          // the tree tile holds every node of the sequence (at most 128) from
+          // key 0: key k of this half is bit k of the half's ancestor word
+          const uint64_t am = tree ? (hf ? ahi : alo) : ~0ull;
 #pragma unroll
           for (int k = 0; k < 64; ++k) {
-            const int key = 64 * hf + k;
-            bool v = key < valid;
-            if (tree) v = v && anc_bit(alo, ahi, key0 + key);
+            const bool v = (64 * hf + k < valid) && ((am >> k) & 1ull);
             xs[k] = v ? xs[k] : -INFINITY;
           }
         }
