@@ -314,7 +314,7 @@ THREAD_VARS = ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS",
                "BLIS_NUM_THREADS", "VECLIB_MAXIMUM_THREADS", "NUMEXPR_NUM_THREADS")
 
 
-def oracle_single_thread(wl):
+def oracle_single_thread(wl, tau=None):
     """One oracle verify step of the same workload on one host core: a child
     process (BLAS threads 1, pinned to one core) redraws the workload from its
     seed, takes the drafted tokens from a file and times one step."""
@@ -324,7 +324,7 @@ def oracle_single_thread(wl):
         np.save(path, wl.tokens)
         env = dict(os.environ, **{v: "1" for v in THREAD_VARS})
         r = subprocess.run([sys.executable, os.path.abspath(__file__), "--oracle-one-step", path,
-                            "--config", str(wl.config), "--tau", repr(TAU)],
+                            "--config", str(wl.config), "--tau", repr(TAU if tau is None else tau)],
                            env=env, capture_output=True, text=True, timeout=900)
         if r.returncode != 0:
             return {"error": (r.stderr or r.stdout).strip().splitlines()[-1:]}
@@ -677,9 +677,29 @@ def workloads_block(device, stream, steps=10, warmup=3):
         }
         del step, out
         torch.cuda.empty_cache()
+    # the tiny fp32 workload (parity case): its step time and the oracle on one core
+    wl = synth.make_workload(1)
+    synth.attach_tokens(wl, ranks_torch(wl, device))
+    tau = synth.WORKLOADS[1]["tau"][0]
+    step, _, _ = device_step(wl, device, tau)
+    for _ in range(warmup):
+        step.run(stream)
+    torch.cuda.synchronize()
+    ms = time_region(step, stream, 10 * steps)
+    out = outputs_numpy(step)
+    single = oracle_single_thread(wl, tau)
+    res[wl.name] = {
+        "config": 1, "batch": wl.B, "tree_nodes": wl.T, "tau": tau, "dtype": "f32",
+        "us_per_step": 1e3 * ms, "value": wl.T / (ms * 1e-3), "unit": UNIT,
+        "steps": 10 * steps, "device_status": step.device_status(),
+        "parity": parity_check(wl, tau, out, cache_reader(wl, step)),
+        "cpu_baseline_single_thread": single,
+    }
+    del step
     return {"note": "tensor-bound workloads, each a short timed loop after the headline "
                     "(burst regime: fractions against the burst bf16 peak); inputs larger than "
-                    "L2 (the LM-head weight is streamed every step)", **res}
+                    "L2 (the LM-head weight is streamed every step); and the tiny fp32 "
+                    "workload with the oracle timed on one core", **res}
 
 
 def run_asd(args):
