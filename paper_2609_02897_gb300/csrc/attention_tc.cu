@@ -7,30 +7,35 @@
 // Work item (one CTA): 128 query rows of one (sequence, KV head) pair, the
 // whole context.  The rows of a pair are its N nodes times the G query heads
 // that share the KV head, node-major (row r -> node r / G, head g*G + r % G);
-// row r lives in TMEM lane r.  Keys come in tiles of 128 through a 3-stage
-// TMA ring (128-byte swizzle; paged caches one box per page; the tree K/V
-// through a 3D map over [T, Hkv, D]); the last tile of a pair holds its tree
-// keys, where a node sees only its ancestors (bitmasks derived here from the
-// parent array).
+// row r lives in TMEM lane r.  Keys come in tiles of 128, K and V through
+// TMA rings of their own (128-byte swizzle; paged caches one box per page;
+// the tree K/V through a 3D map over [T, Hkv, D]), so a K slot is refilled
+// as soon as its S MMA is done rather than after the tile's P.V; the
+// last tile of a pair holds its tree keys, where a node sees only its
+// ancestors (bitmasks derived here from the parent array).
 //
-//   Q             staged once into TMEM by the softmax warps
-//   S = Q . K^T   tcgen05.mma, A (= Q) from TMEM, K K-major in shared memory
+//   Q             staged once into shared memory by the softmax warps
+//   S = Q . K^T   tcgen05.mma, Q and K K-major in shared memory
 //   P = exp2(S*c - m), per row by the thread that owns the row, written back
 //                 over the tile's S columns as bf16 pairs
 //   O += P . V    tcgen05.mma, A (= P) from TMEM, V MN-major straight from its
 //                 TMA tile, O in TMEM for the whole item
 //
-// Every MMA thus reads one operand from shared memory.  The softmax keeps a
+// The softmax keeps a
 // per-row reference max m and rescales O only when the running max exceeds m
 // by more than 2^8 in the exp2 domain (P then stays below 2^8 and the result
-// equals that with the exact running max).  S/P is double-buffered: the MMAs
-// of tile t+1 run while the softmax works on tile t.
+// equals that with the exact running max).  S/P is triple-buffered: S of tile
+// t+1 is ready when the softmax finishes tile t, and S of tile t+2 does not
+// wait for O += P V of tile t (with two buffers it did, which put the P.V,
+// its commit and the next S on the softmax's path every second tile).
 //
-// TMEM (512 columns): O [0, D), Q [128, 128 + D/2), S/P [256, 384) and
-// [384, 512).  Shared memory: the K/V ring, 3 x 64 KB for D = 128.
-// Warp roles (320 threads): warp 0 TMA producer, warp 1 TMEM allocator and
-// MMA issuer, warps 2-9 softmax and epilogue, two per TMEM lane quarter, each
-// on one half of every tile's keys.
+// TMEM (512 columns): O [0, D), S/P [128, 256), [256, 384), [384, 512).
+// Shared memory: Q, a 3-stage K ring and a V ring (160 KB of rings for D =
+// 128).
+// Warp roles (384 threads): warp 0 K producer, warp 1 TMEM allocator and
+// issuer of the S MMAs, warps 2-9 softmax and epilogue, two per TMEM lane
+// quarter, each on one half of every tile's keys, warp 10 issuer of the P.V
+// MMAs, warp 11 V producer.
 #include "kernels.h"
 #include "tc.cuh"
 
@@ -39,23 +44,27 @@ namespace {
 
 constexpr int kRows = kAttnTcRows;   // query rows per CTA = TMEM lanes
 constexpr int kKeys = kAttnTcKeys;   // keys per tile
-constexpr int kStages = 3;           // K/V ring
-constexpr int kThreads = 320;
+constexpr int kThreads = 320;     // ping-pong kernel
+constexpr int kTcThreads = 384;   // one-tile kernel: twelve warps
 constexpr int kSoftmaxThreads = 256;   // eight warps: two per TMEM lane quarter
 constexpr float kRescaleLog2 = 8.f;
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kQCol = 128;
-constexpr uint32_t kSCol0 = 256;
+constexpr int kSBufs = 3;              // S/P buffers in TMEM
+constexpr uint32_t kSCol0 = 128;       // S/P buffer b at columns [128 (b + 1), 128 (b + 2))
 
-// Dynamic shared memory, 1024-byte aligned: K [stage][D/64][128 keys][128 B],
-// then V likewise.
+// Dynamic shared memory, 1024-byte aligned: Q [D/64][128 rows][128 B], the K
+// ring [stage][D/64][128 keys][128 B], then the V ring likewise (two stages
+// for D = 128, where a third does not fit beside Q).
 template <int D>
 struct TcGeom {
   static constexpr int kNH = D / 64;
   static constexpr int kTileBytes = kNH * kKeys * 128;   // one K or one V tile
-  static constexpr int kKOff = 0;
-  static constexpr int kVOff = kStages * kTileBytes;
-  static constexpr int kBytes = kVOff + kStages * kTileBytes;
+  static constexpr int kKStages = 3;
+  static constexpr int kVStages = D == 64 ? 3 : 2;
+  static constexpr int kQOff = 0;
+  static constexpr int kKOff = kNH * kRows * 128;
+  static constexpr int kVOff = kKOff + kKStages * kTileBytes;
+  static constexpr int kBytes = kVOff + kVStages * kTileBytes;
 };
 
 // Named barrier 1 of the eight softmax warps.
@@ -132,52 +141,44 @@ __device__ __forceinline__ size_t grow_of(const AttnParams& p, const Item& it, i
   return static_cast<size_t>(it.s0 + i) * p.Hq + it.g * p.G + (rr - i * p.G);
 }
 
-// Issues the K and V tiles of a contiguous-cache or tree tile t into one
-// stage (producer lane 0 only).
+constexpr int kPageChunk = 512;   // page-table entries staged in shared memory
+
+// Issues one K (which = 0) or V (which = 1) tile t into `dst` (producer lane 0;
+// contiguous cache or tree keys).
 template <int D>
-__device__ __forceinline__ void issue_tile(const AttnParams& p, const Item& it, int t,
-                                           uint32_t k_s, uint32_t v_s, uint32_t bar,
-                                           const CUtensorMap* tm_k, const CUtensorMap* tm_v,
-                                           const CUtensorMap* tm_tk, const CUtensorMap* tm_tv,
-                                           uint64_t pol) {
+__device__ __forceinline__ void issue_half_tile(const AttnParams& p, const Item& it, int t,
+                                                uint32_t dst, uint32_t bar,
+                                                const CUtensorMap* tm, const CUtensorMap* tm_tree,
+                                                uint64_t pol) {
   using G = TcGeom<D>;
-  mbar_expect_tx(bar, 2 * G::kTileBytes);
+  mbar_expect_tx(bar, G::kTileBytes);
   if (t >= it.nctx) {
-    // tree keys: rows s0 + key0 .. of KV head g (rows past T read as zeros)
     const int key0 = (t - it.nctx) * kKeys;
 #pragma unroll
-    for (int h = 0; h < G::kNH; ++h) {
-      tma_load_3d(k_s + h * (kKeys * 128), tm_tk, bar, h * 64, it.g, it.s0 + key0, pol);
-      tma_load_3d(v_s + h * (kKeys * 128), tm_tv, bar, h * 64, it.g, it.s0 + key0, pol);
-    }
+    for (int h = 0; h < G::kNH; ++h)
+      tma_load_3d(dst + h * (kKeys * 128), tm_tree, bar, h * 64, it.g, it.s0 + key0, pol);
     return;
   }
   const int row = (it.b * p.Hkv + it.g) * p.ctx_max + t * kKeys;
 #pragma unroll
-  for (int h = 0; h < G::kNH; ++h) {
-    tma_load_2d(k_s + h * (kKeys * 128), tm_k, bar, h * 64, row, pol);
-    tma_load_2d(v_s + h * (kKeys * 128), tm_v, bar, h * 64, row, pol);
-  }
+  for (int h = 0; h < G::kNH; ++h) tma_load_2d(dst + h * (kKeys * 128), tm, bar, h * 64, row, pol);
 }
 
-constexpr int kPageChunk = 512;   // page-table entries staged in shared memory
-
-// Issues the K and V boxes of paged context tile t into one stage (the whole
-// producer warp): one box of min(page, 128) rows per page the tile touches,
-// lane j taking page j of the tile, its page id read from a chunk of the
-// sequence's page-table row that the warp stages in shared memory (`chunk0`:
-// first staged entry, -1 before the first chunk).  Pages past the context
-// are not loaded; an out-of-range page id is reported and not loaded.
+// Paged context tile t, K or V (the whole producer warp): one box of
+// min(page, 128) rows per page the tile touches, lane j taking page j of the
+// tile, its page id read from a chunk of the sequence's page-table row that
+// the warp stages in shared memory (`chunk0`: first staged entry, -1 before
+// the first chunk).  Pages past the context are not loaded; an out-of-range
+// page id is reported and not loaded.
 template <int D>
-__device__ __forceinline__ void issue_paged_tile(const AttnParams& p, const Item& it, int t,
-                                                 uint32_t k_s, uint32_t v_s, uint32_t bar,
-                                                 const CUtensorMap* tm_k, const CUtensorMap* tm_v,
+__device__ __forceinline__ void issue_paged_half(const AttnParams& p, const Item& it, int t,
+                                                 uint32_t dst, uint32_t bar, const CUtensorMap* tm,
                                                  uint64_t pol, int* s_pages, int& chunk0,
                                                  int lane) {
   using G = TcGeom<D>;
   const int ps = p.page_size;
   const int br = ps < kKeys ? ps : kKeys;
-  const int nbox = kKeys / br;   // <= 16 (pages hold at least 8 rows)
+  const int nbox = kKeys / br;
   const int key0 = t * kKeys;
   const int e_first = key0 / ps, e_last = (key0 + (nbox - 1) * br) / ps;
   if (chunk0 < 0 || e_first < chunk0 || e_last >= chunk0 + kPageChunk) {
@@ -201,15 +202,12 @@ __device__ __forceinline__ void issue_paged_tile(const AttnParams& p, const Item
     }
   }
   const uint32_t valid = __ballot_sync(0xffffffffu, row >= 0);
-  if (lane == 0)
-    mbar_expect_tx(bar, static_cast<uint32_t>(__popc(valid) * 2 * G::kNH * br * 128));
+  if (lane == 0) mbar_expect_tx(bar, static_cast<uint32_t>(__popc(valid) * G::kNH * br * 128));
   __syncwarp();
   if (row >= 0) {
 #pragma unroll
-    for (int h = 0; h < G::kNH; ++h) {
-      tma_load_2d(k_s + h * (kKeys * 128) + lane * br * 128, tm_k, bar, h * 64, row, pol);
-      tma_load_2d(v_s + h * (kKeys * 128) + lane * br * 128, tm_v, bar, h * 64, row, pol);
-    }
+    for (int h = 0; h < G::kNH; ++h)
+      tma_load_2d(dst + h * (kKeys * 128) + lane * br * 128, tm, bar, h * 64, row, pol);
   }
   __syncwarp();
 }
@@ -230,8 +228,8 @@ __device__ __forceinline__ bool softmax_role(const AttnParams& p, const Item& it
                                              float (*s_mx)[2][kRows], float (*s_l)[kRows],
                                              uint64_t* q_ready, uint64_t* s_full,
                                              uint64_t* p_full, uint64_t* pv_done,
-                                             volatile int* s_abort, long long budget,
-                                             float& inv) {
+                                             uint64_t* v_full, volatile int* s_abort,
+                                             long long budget, float& inv) {
   using G = TcGeom<D>;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int hf = (warp - 2) >> 2;              // key half of every tile
@@ -239,28 +237,22 @@ __device__ __forceinline__ bool softmax_role(const AttnParams& p, const Item& it
   const int tid = threadIdx.x - 64;            // 0..255
   const uint32_t lane_base = tmem + (static_cast<uint32_t>((warp & 3) * 32) << 16);
 
-  // this half of the row's query -> TMEM columns kQCol + [hf D/4, (hf+1) D/4),
-  // bf16 pairs; zeros past nrows
+  // this half of the row's query (16-byte chunks [hf D/16, (hf+1) D/16)) ->
+  // shared memory, 128-byte swizzled like a TMA tile; zeros past nrows
   {
     const bool mine = row < it.nrows;
     const uint4* qg = reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(p.q) +
-                                                     (mine ? grow_of(p, it, row) : 0) * D +
-                                                     hf * (D / 2));
+                                                     (mine ? grow_of(p, it, row) : 0) * D);
+    uint8_t* qs = gbase + G::kQOff;
 #pragma unroll
-    for (int c = 0; c < D / 64; ++c) {
-      uint32_t r[16];
-#pragma unroll
-      for (int k = 0; k < 4; ++k) {
-        const uint4 v = mine ? qg[c * 4 + k] : make_uint4(0u, 0u, 0u, 0u);
-        r[4 * k] = v.x;
-        r[4 * k + 1] = v.y;
-        r[4 * k + 2] = v.z;
-        r[4 * k + 3] = v.w;
-      }
-      tmem_st16(lane_base + kQCol + hf * (D / 4) + 16 * c, r);
+    for (int k = 0; k < D / 16; ++k) {
+      const int c = hf * (D / 16) + k;
+      const uint4 v = mine ? qg[c] : make_uint4(0u, 0u, 0u, 0u);
+      *reinterpret_cast<uint4*>(qs + (c >> 3) * (kRows * 128) + row * 128 +
+                                (((c & 7) ^ (row & 7)) << 4)) = v;
     }
   }
-  tc_fence_before();
+  fence_proxy_async();   // the tensor cores read these rows
   __syncwarp();
   if (lane == 0) mbar_arrive(smem_u32(q_ready));
 
@@ -274,14 +266,15 @@ __device__ __forceinline__ bool softmax_role(const AttnParams& p, const Item& it
   float m_ref = -INFINITY, l = 0.f;
   bool ok = true, bad = false;
   for (int t = 0; t < it.ntiles; ++t) {
-    const int b = t & 1;
+    const int b = t % kSBufs, e = t & 1;
     const uint32_t sb = lane_base + kSCol0 + b * kKeys;
     const bool tree = t >= it.nctx;
     const int key0 = tree ? (t - it.nctx) * kKeys : t * kKeys;
     const int valid = min(kKeys, (tree ? it.n : it.ctx) - key0);
     float x[64];
     float mt = -INFINITY;
-    const bool here = !bad && wait_all(&s_full[b], (t >> 1) & 1, budget) && !aborted_warp(s_abort);
+    const bool here =
+        !bad && wait_all(&s_full[b], (t / kSBufs) & 1, budget) && !aborted_warp(s_abort);
     if (here) {
       tc_fence_after();
       tmem_ld64(sb + 64 * hf, x);
@@ -297,14 +290,14 @@ __device__ __forceinline__ bool softmax_role(const AttnParams& p, const Item& it
       }
 #pragma unroll
       for (int k = 0; k < 64; ++k) mt = fmaxf(mt, x[k]);
-      s_mx[b][hf][row] = mt;
+      s_mx[e][hf][row] = mt;
     }
     // every softmax warp decides together whether to go on (no warp may be
     // left waiting at a barrier), and the partial maxima become visible
     ok = softmax_all(here);
     if (!ok) break;
     // the row's max over both halves (raw scores; the scale is positive)
-    mt = fmaxf(mt, s_mx[b][hf ^ 1][row]) * c;
+    mt = fmaxf(mt, s_mx[e][hf ^ 1][row]) * c;
     const float mn = fmaxf(m_ref, mt);
     const bool had = m_ref != -INFINITY;
     const bool need = had ? (mn > m_ref + kRescaleLog2) : (mn != -INFINITY);
@@ -312,7 +305,7 @@ __device__ __forceinline__ bool softmax_role(const AttnParams& p, const Item& it
       // O holds earlier tiles of this row: rescale this half of it once
       // O += P V of tile t-1 is done
       // (a wait that gives up marks the thread; all leave at the next tile)
-      if (!wait_all(&pv_done[(t - 1) & 1], ((t - 1) >> 1) & 1, budget)) {
+      if (!wait_all(&pv_done[(t - 1) % kSBufs], ((t - 1) / kSBufs) & 1, budget)) {
         bad = true;
       } else {
         tc_fence_after();
@@ -344,23 +337,31 @@ __device__ __forceinline__ bool softmax_role(const AttnParams& p, const Item& it
     tmem_st32u(sb + 32 * hf, pk);
     if (valid < kKeys) {
       // ragged tile: V rows past the last valid key may hold anything; zero
-      // them so that 0 * V stays 0
-      uint8_t* vt = gbase + G::kVOff + (t % kStages) * G::kTileBytes;
-      constexpr int kChunksPerRow = G::kNH * 8;
-      for (int i = tid; i < (kKeys - valid) * kChunksPerRow; i += kSoftmaxThreads) {
-        const int r = valid + i / kChunksPerRow, rem = i % kChunksPerRow;
-        *reinterpret_cast<uint4*>(vt + (rem >> 3) * (kKeys * 128) + r * 128 + (rem & 7) * 16) =
-            make_uint4(0u, 0u, 0u, 0u);
+      // them so that 0 * V stays 0, once the V tile has landed (it comes
+      // through its own ring and may still be in flight)
+      if (!bad && wait_all(&v_full[t % G::kVStages], (t / G::kVStages) & 1, budget)) {
+        uint8_t* vt = gbase + G::kVOff + (t % G::kVStages) * G::kTileBytes;
+        constexpr int kChunksPerRow = G::kNH * 8;
+        for (int i = tid; i < (kKeys - valid) * kChunksPerRow; i += kSoftmaxThreads) {
+          const int r = valid + i / kChunksPerRow, rem = i % kChunksPerRow;
+          *reinterpret_cast<uint4*>(vt + (rem >> 3) * (kKeys * 128) + r * 128 + (rem & 7) * 16) =
+              make_uint4(0u, 0u, 0u, 0u);
+        }
+        fence_proxy_async();  // the zeroed rows are read by the tensor cores
+      } else {
+        bad = true;
       }
-      fence_proxy_async();  // the zeroed rows are read by the tensor cores
     }
     tc_fence_before();
     __syncwarp();
     if (lane == 0) mbar_arrive(smem_u32(&p_full[b]));
   }
   if (ok) {
+    // O is complete once the last P.V is done (S of the last tile waited for
+    // the P.V three tiles back, so that buffer's pending phase is the last's)
     const int last = it.ntiles - 1;
-    ok = !bad && wait_all(&pv_done[last & 1], (last >> 1) & 1, budget) && !aborted_warp(s_abort);
+    ok = !bad && wait_all(&pv_done[last % kSBufs], (last / kSBufs) & 1, budget) &&
+         !aborted_warp(s_abort);
     if (ok) tc_fence_after();
   }
   if (softmax_any(!ok)) {
@@ -379,26 +380,28 @@ __device__ __forceinline__ bool softmax_role(const AttnParams& p, const Item& it
 }
 
 template <int D>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(kTcThreads, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_v,
                    const __grid_constant__ CUtensorMap tm_tk,
                    const __grid_constant__ CUtensorMap tm_tv, const AttnParams p) {
   using G = TcGeom<D>;
   extern __shared__ uint8_t smem_raw[];
-  __shared__ __align__(8) uint64_t s_kv_full[kStages];
-  __shared__ __align__(8) uint64_t s_kv_empty[kStages];
-  __shared__ __align__(8) uint64_t s_s_full[2];    // S of a tile in TMEM (MMA -> softmax)
-  __shared__ __align__(8) uint64_t s_p_full[2];    // P of a tile in TMEM (softmax -> MMA)
-  __shared__ __align__(8) uint64_t s_pv_done[2];   // O += P V of a tile done (MMA -> softmax)
+  constexpr int KS = G::kKStages, VS = G::kVStages;
+  __shared__ __align__(8) uint64_t s_k_full[KS], s_k_empty[KS];
+  __shared__ __align__(8) uint64_t s_v_full[VS], s_v_empty[VS];
+  __shared__ __align__(8) uint64_t s_s_full[kSBufs];    // S of a tile in TMEM (MMA -> softmax)
+  __shared__ __align__(8) uint64_t s_p_full[kSBufs];    // P of a tile in TMEM (softmax -> MMA)
+  __shared__ __align__(8) uint64_t s_pv_done[kSBufs];   // O += P V of a tile done (MMA -> softmax)
   __shared__ __align__(8) uint64_t s_q_ready;
-  __shared__ __align__(8) uint64_t s_mma_done;
+  __shared__ __align__(8) uint64_t s_mma_done[2];   // each MMA issuer's own drain
   __shared__ uint32_t s_tmem;
   __shared__ volatile int s_abort;
   __shared__ int s_par[kMaxNodes];
   __shared__ uint64_t s_anc[kMaxNodes][2];
   __shared__ float s_mx[2][2][kRows];   // [tile parity][key half][row]: partial row max
   __shared__ float s_l[2][kRows];       // [key half][row]: partial row sum
-  __shared__ int s_pages[kPageChunk];   // producer: staged page-table entries (paged caches)
+  __shared__ int s_pages[2][kPageChunk];   // K / V producer: staged page-table entries
+  __shared__ int s_issued[2][KS > VS ? KS : VS];  // producer: K (0) / V (1) fills per stage
 
   pdl_launch_dependents();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -413,20 +416,27 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t pad = (1024u - (base & 1023u)) & 1023u;
   uint8_t* gbase = smem_raw + pad;
   base += pad;
-  const uint32_t k_s0 = base + G::kKOff, v_s0 = base + G::kVOff;
+  const uint32_t q_s = base + G::kQOff, k_s0 = base + G::kKOff, v_s0 = base + G::kVOff;
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < kStages; ++s) {
-      mbar_init(smem_u32(&s_kv_full[s]), 1);
-      mbar_init(smem_u32(&s_kv_empty[s]), 1);
+    for (int s = 0; s < KS; ++s) {
+      mbar_init(smem_u32(&s_k_full[s]), 1);
+      mbar_init(smem_u32(&s_k_empty[s]), 1);
+      s_issued[0][s] = 0;
     }
-    for (int b = 0; b < 2; ++b) {
+    for (int s = 0; s < VS; ++s) {
+      mbar_init(smem_u32(&s_v_full[s]), 1);
+      mbar_init(smem_u32(&s_v_empty[s]), 1);
+      s_issued[1][s] = 0;
+    }
+    for (int b = 0; b < kSBufs; ++b) {
       mbar_init(smem_u32(&s_s_full[b]), 1);
       mbar_init(smem_u32(&s_p_full[b]), kSoftmaxThreads / 32);
       mbar_init(smem_u32(&s_pv_done[b]), 1);
     }
     mbar_init(smem_u32(&s_q_ready), kSoftmaxThreads / 32);
-    mbar_init(smem_u32(&s_mma_done), 1);
+    mbar_init(smem_u32(&s_mma_done[0]), 1);
+    mbar_init(smem_u32(&s_mma_done[1]), 1);
     s_abort = 0;
     fence_mbar_init();
   }
@@ -436,9 +446,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   // ancestor bitmasks (self included) of the sequence's nodes for the tree
   // tile; a malformed parent ends the walk, so it is bounded
-  for (int i = threadIdx.x; i < it.n; i += kThreads) s_par[i] = p.parent[it.s0 + i];
+  for (int i = threadIdx.x; i < it.n; i += kTcThreads) s_par[i] = p.parent[it.s0 + i];
   __syncthreads();
-  for (int i = threadIdx.x; i < it.n; i += kThreads) {
+  for (int i = threadIdx.x; i < it.n; i += kTcThreads) {
     uint64_t lo = 0, hi = 0;
     int u = i;
     while (true) {
@@ -457,70 +467,87 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   bool ok = false;           // softmax warps: O complete in TMEM
   float inv = 0.f;
-  if (warp == 0) {
-    // ------------------------------------------------------------ TMA producer
+  if (warp == 0 || warp == 11) {
+    // ----------------------------------------------------------- TMA producers
+    // K and V come through rings of their own, each filled by its own warp
+    // (warp 0 K, warp 11 V), so that neither ring waits behind the other: a K
+    // slot is free again once the S MMA of its tile is done, a V slot once the
+    // P.V MMA is.
+    const int which = warp == 0 ? 0 : 1;
+    const int ns = which ? VS : KS;
     if (lane == 0) {
-      prefetch_tmap(&tm_k);
-      prefetch_tmap(&tm_v);
-      prefetch_tmap(&tm_tk);
-      prefetch_tmap(&tm_tv);
+      prefetch_tmap(which ? &tm_v : &tm_k);
+      prefetch_tmap(which ? &tm_tv : &tm_tk);
     }
     const uint64_t pol = l2_policy_evict_first();
-    int issued = 0;
     int chunk0 = -1;
-    for (int t = 0; t < it.ntiles; ++t) {
-      const int stage = t % kStages;
-      if (!wait_all(&s_kv_empty[stage], ((t / kStages) & 1) ^ 1u, budget)) {
-        if (lane == 0) {
-          note_timeout(p.status);
-          s_abort = 1;
-        }
+    bool pok = true;
+    for (int t = 0; pok && t < it.ntiles; ++t) {
+      const int stage = t % ns;
+      uint64_t* empty = which ? &s_v_empty[stage] : &s_k_empty[stage];
+      uint64_t* full = which ? &s_v_full[stage] : &s_k_full[stage];
+      if (!wait_all(empty, ((t / ns) & 1) ^ 1u, budget) || aborted_warp(&s_abort)) {
+        pok = false;
         break;
       }
-      if (aborted_warp(&s_abort)) break;
-      const uint32_t k_st = k_s0 + stage * G::kTileBytes, v_st = v_s0 + stage * G::kTileBytes;
+      const uint32_t dst = base + (which ? G::kVOff : G::kKOff) + stage * G::kTileBytes;
       if (p.page_size != 0 && t < it.nctx)
-        issue_paged_tile<D>(p, it, t, k_st, v_st, smem_u32(&s_kv_full[stage]), &tm_k, &tm_v, pol,
-                            s_pages, chunk0, lane);
+        issue_paged_half<D>(p, it, t, dst, smem_u32(full), which ? &tm_v : &tm_k, pol,
+                            s_pages[which], chunk0, lane);
       else if (lane == 0)
-        issue_tile<D>(p, it, t, k_st, v_st, smem_u32(&s_kv_full[stage]), &tm_k, &tm_v, &tm_tk,
-                      &tm_tv, pol);
+        issue_half_tile<D>(p, it, t, dst, smem_u32(full), which ? &tm_v : &tm_k,
+                           which ? &tm_tv : &tm_tk, pol);
+      if (lane == 0) ++s_issued[which][stage];
       __syncwarp();
-      ++issued;
+    }
+    if (!pok && lane == 0) {
+      note_timeout(p.status);
+      s_abort = 1;
     }
     // every copy issued has landed before the buffers are reused or left
     if (lane == 0)
-      for (int t = max(0, issued - kStages); t < issued; ++t)
-        mbar_wait(smem_u32(&s_kv_full[t % kStages]), (t / kStages) & 1);
+      for (int st = 0; st < ns; ++st)
+        if (s_issued[which][st] > 0)
+          mbar_wait(smem_u32(which ? &s_v_full[st] : &s_k_full[st]),
+                    static_cast<uint32_t>((s_issued[which][st] - 1) & 1));
     __syncwarp();
-  } else if (warp == 1) {
-    // --------------------------------------------------------------- MMA issuer
+  } else if (warp == 1 || warp == 10) {
+    // ------------------------------------------------------------ MMA issuers
+    // Two issuing threads, so that the one's barrier waits (each a few hundred
+    // cycles even on a completed phase) overlap the other's MMAs: warp 1
+    // issues S = Q K^T of every tile, warp 10 O += P V.  Each commit tracks the
+    // issuing thread's own MMAs.
     if (lane == 0) {
-      const uint32_t idesc_s = idesc_bf16(kRows, kKeys);         // S = Q K^T
-      const uint32_t idesc_o = idesc_bf16(kRows, D, true);       // O += P V, V MN-major
-      bool mok = mbar_wait(smem_u32(&s_q_ready), 0, budget);
-      if (mok) tc_fence_after();
-      for (int t = 0; mok && t <= it.ntiles; ++t) {
-        if (t < it.ntiles) {
-          const int stage = t % kStages, b = t & 1;
-          mok = mbar_wait(smem_u32(&s_kv_full[stage]), (t / kStages) & 1, budget);
-          // the S/P buffer is free once O += P V of tile t-2 is done
-          if (mok && t >= 2) mok = mbar_wait(smem_u32(&s_pv_done[b]), ((t >> 1) - 1) & 1, budget);
+      bool mok = true;
+      if (warp == 1) {
+        const uint32_t idesc_s = idesc_bf16(kRows, kKeys);   // S = Q K^T
+        mok = mbar_wait(smem_u32(&s_q_ready), 0, budget);
+        if (mok) tc_fence_after();
+        for (int t = 0; mok && t < it.ntiles; ++t) {
+          const int stage = t % KS, b = t % kSBufs;
+          mok = mbar_wait(smem_u32(&s_k_full[stage]), (t / KS) & 1, budget);
+          // the S/P buffer is free once O += P V of tile t-3 is done
+          if (mok && t >= kSBufs)
+            mok = mbar_wait(smem_u32(&s_pv_done[b]), ((t / kSBufs) - 1) & 1, budget);
           if (!mok || s_abort) break;
           tc_fence_after();
           const uint32_t kst = k_s0 + stage * G::kTileBytes;
 #pragma unroll
           for (int ks = 0; ks < D / 16; ++ks) {
             const int h = ks >> 2, kk = ks & 3;
-            tc_mma_ts(tmem + kSCol0 + b * kKeys, tmem + kQCol + ks * 8,
-                      sw128_desc(kst + h * (kKeys * 128) + 32 * kk), idesc_s, ks > 0 ? 1u : 0u);
+            tc_mma(tmem + kSCol0 + b * kKeys, sw128_desc(q_s + h * (kRows * 128) + 32 * kk),
+                   sw128_desc(kst + h * (kKeys * 128) + 32 * kk), idesc_s, ks > 0 ? 1u : 0u);
           }
           tc_commit(smem_u32(&s_s_full[b]));
+          tc_commit(smem_u32(&s_k_empty[stage]));
         }
-        if (t >= 1) {
-          // O += P_j V_j for the previous tile j, after its softmax
-          const int j = t - 1, stage = j % kStages, b = j & 1;
-          mok = mbar_wait(smem_u32(&s_p_full[b]), (j >> 1) & 1, budget);
+      } else {
+        const uint32_t idesc_o = idesc_bf16(kRows, D, true);   // O += P V, V MN-major
+        for (int j = 0; mok && j < it.ntiles; ++j) {
+          // O += P_j V_j once tile j's softmax has written P_j
+          const int stage = j % VS, b = j % kSBufs;
+          mok = mbar_wait(smem_u32(&s_p_full[b]), (j / kSBufs) & 1, budget) &&
+                mbar_wait(smem_u32(&s_v_full[stage]), (j / VS) & 1, budget);
           if (!mok || s_abort) break;
           tc_fence_after();
           const uint32_t vst = v_s0 + stage * G::kTileBytes;
@@ -530,28 +557,30 @@ __global__ void __launch_bounds__(kThreads, 1)
                       sw128_desc_mn(vst + kk * 2048, kKeys * 128, 1024), idesc_o,
                       (j > 0 || kk > 0) ? 1u : 0u);
           tc_commit(smem_u32(&s_pv_done[b]));
-          tc_commit(smem_u32(&s_kv_empty[stage]));
+          tc_commit(smem_u32(&s_v_empty[stage]));
         }
       }
       if (!mok) {
         note_timeout(p.status);
         s_abort = 1;
       }
-      // every MMA issued above has finished before TMEM or the buffers are reused
-      tc_commit(smem_u32(&s_mma_done));
-      mbar_wait(smem_u32(&s_mma_done), 0);
+      // every MMA this thread issued has finished before TMEM or the buffers
+      // are reused
+      uint64_t* done = &s_mma_done[warp == 1 ? 0 : 1];
+      tc_commit(smem_u32(done));
+      mbar_wait(smem_u32(done), 0);
     }
     __syncwarp();
   } else {
     ok = softmax_role<D>(p, it, tmem, gbase, s_anc, s_mx, s_l, &s_q_ready, s_s_full, s_p_full,
-                         s_pv_done, &s_abort, budget, inv);
+                         s_pv_done, s_v_full, &s_abort, budget, inv);
   }
 
   // ------------------------------------------------------------------ finish
   tc_fence_before();
   __syncthreads();   // the tile buffers and the tensor cores are idle from here on
   tc_fence_after();
-  if (warp >= 2 && ok) {
+  if (warp >= 2 && warp < 10 && ok) {
     // each thread writes its key half's share of the row: D/2 output columns
     const int hf = (warp - 2) >> 2;
     const int row = (warp & 3) * 32 + lane;   // TMEM lane = query row
@@ -632,70 +661,6 @@ __device__ __forceinline__ bool make_item_pp(const AttnParams& p, Item& it) {
   it.ntree = (it.n + kKeys - 1) / kKeys;
   it.ntiles = it.nctx + it.ntree;
   return true;
-}
-
-// Issues one K (which = 0) or V (which = 1) tile t into `dst` (producer lane 0;
-// contiguous cache or tree keys).
-template <int D>
-__device__ __forceinline__ void issue_half_tile(const AttnParams& p, const Item& it, int t,
-                                                uint32_t dst, uint32_t bar,
-                                                const CUtensorMap* tm, const CUtensorMap* tm_tree,
-                                                uint64_t pol) {
-  using G = PPGeom<D>;
-  mbar_expect_tx(bar, G::kKVTile);
-  if (t >= it.nctx) {
-    const int key0 = (t - it.nctx) * kKeys;
-#pragma unroll
-    for (int h = 0; h < G::kNH; ++h)
-      tma_load_3d(dst + h * (kKeys * 128), tm_tree, bar, h * 64, it.g, it.s0 + key0, pol);
-    return;
-  }
-  const int row = (it.b * p.Hkv + it.g) * p.ctx_max + t * kKeys;
-#pragma unroll
-  for (int h = 0; h < G::kNH; ++h) tma_load_2d(dst + h * (kKeys * 128), tm, bar, h * 64, row, pol);
-}
-
-// Paged context tile t, K or V (the whole producer warp; see issue_paged_tile).
-template <int D>
-__device__ __forceinline__ void issue_paged_half(const AttnParams& p, const Item& it, int t,
-                                                 uint32_t dst, uint32_t bar, const CUtensorMap* tm,
-                                                 uint64_t pol, int* s_pages, int& chunk0,
-                                                 int lane) {
-  using G = PPGeom<D>;
-  const int ps = p.page_size;
-  const int br = ps < kKeys ? ps : kKeys;
-  const int nbox = kKeys / br;
-  const int key0 = t * kKeys;
-  const int e_first = key0 / ps, e_last = (key0 + (nbox - 1) * br) / ps;
-  if (chunk0 < 0 || e_first < chunk0 || e_last >= chunk0 + kPageChunk) {
-    chunk0 = e_first;
-    const int32_t* row_pt = p.page_table + static_cast<size_t>(it.b) * p.pages_per_seq;
-    for (int i = lane; i < kPageChunk; i += 32) {
-      const int e = chunk0 + i;
-      s_pages[i] = e < p.pages_per_seq ? row_pt[e] : -1;
-    }
-    __syncwarp();
-  }
-  int row = -1;
-  if (lane < nbox) {
-    const int key = key0 + lane * br;
-    if (key < it.ctx) {
-      const int page = s_pages[key / ps - chunk0];
-      if (page < 0 || page >= p.num_pages)
-        set_status(p.status, ASD_ERR_CTX_RANGE);
-      else
-        row = (page * p.Hkv + it.g) * ps + (key % ps);
-    }
-  }
-  const uint32_t valid = __ballot_sync(0xffffffffu, row >= 0);
-  if (lane == 0) mbar_expect_tx(bar, static_cast<uint32_t>(__popc(valid) * G::kNH * br * 128));
-  __syncwarp();
-  if (row >= 0) {
-#pragma unroll
-    for (int h = 0; h < G::kNH; ++h)
-      tma_load_2d(dst + h * (kKeys * 128) + lane * br * 128, tm, bar, h * 64, row, pol);
-  }
-  __syncwarp();
 }
 
 template <int D>
@@ -1113,7 +1078,7 @@ cudaError_t launch_attention_tc(const AttnParams& p, const CUtensorMap& tm_k,
   auto* k = p.D == 64 ? attn_tc_kernel<64> : attn_tc_kernel<128>;
   err = set_smem_attrs(k, smem);
   if (err != cudaSuccess) return err;
-  return launch_pdl(k, grid, dim3(kThreads), smem, s, tm_k, tm_v, tm_tk, tm_tv, p);
+  return launch_pdl(k, grid, dim3(kTcThreads), smem, s, tm_k, tm_v, tm_tk, tm_tv, p);
 }
 
 }  // namespace asd
