@@ -44,8 +44,7 @@ namespace {
 
 constexpr int kRows = kAttnTcRows;   // query rows per CTA = TMEM lanes
 constexpr int kKeys = kAttnTcKeys;   // keys per tile
-constexpr int kThreads = 320;     // ping-pong kernel
-constexpr int kTcThreads = 384;   // one-tile kernel: twelve warps
+constexpr int kThreads = 384;   // twelve warps (roles below)
 constexpr int kSoftmaxThreads = 256;   // eight warps: two per TMEM lane quarter
 constexpr float kRescaleLog2 = 8.f;
 constexpr uint32_t kTmemCols = 512;
@@ -380,7 +379,7 @@ __device__ __forceinline__ bool softmax_role(const AttnParams& p, const Item& it
 }
 
 template <int D>
-__global__ void __launch_bounds__(kTcThreads, 1)
+__global__ void __launch_bounds__(kThreads, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_v,
                    const __grid_constant__ CUtensorMap tm_tk,
                    const __grid_constant__ CUtensorMap tm_tv, const AttnParams p) {
@@ -446,9 +445,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   }
   // ancestor bitmasks (self included) of the sequence's nodes for the tree
   // tile; a malformed parent ends the walk, so it is bounded
-  for (int i = threadIdx.x; i < it.n; i += kTcThreads) s_par[i] = p.parent[it.s0 + i];
+  for (int i = threadIdx.x; i < it.n; i += kThreads) s_par[i] = p.parent[it.s0 + i];
   __syncthreads();
-  for (int i = threadIdx.x; i < it.n; i += kTcThreads) {
+  for (int i = threadIdx.x; i < it.n; i += kThreads) {
     uint64_t lo = 0, hi = 0;
     int u = i;
     while (true) {
@@ -626,8 +625,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 // swizzled, written by the softmax threads); TMEM holds O_A [0, D),
 // O_B [D, 2D) and S/P_A [256, 384), S/P_B [384, 512).  K and V come through
 // separate rings with their own barriers, so a K slot is refilled as soon as
-// both S MMAs have read it.  Warps: 0 TMA producer, 1 MMA issuer (lane 0),
-// 2-5 softmax of tile A, 6-9 softmax of tile B; a softmax thread owns one row
+// both S MMAs have read it.  Warps: 0 K producer, 1 S-MMA issuer (lane 0),
+// 2-5 softmax of tile A, 6-9 softmax of tile B, 10 P.V-MMA issuer (lane 0),
+// 11 V producer; a softmax thread owns one row
 // of its tile and all 128 keys of every key tile, so no exchange between warps
 // is needed: per key tile it reads S twice (the row max, then the
 // exponentials) and writes P as bf16 pairs over the S columns already read.
@@ -676,12 +676,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   __shared__ __align__(8) uint64_t s_p_full[2];    // P of tile X written (softmax X -> MMA)
   __shared__ __align__(8) uint64_t s_pv_done[2];   // O_X += P_X V done (MMA -> softmax X)
   __shared__ __align__(8) uint64_t s_q_ready;
-  __shared__ __align__(8) uint64_t s_mma_done;
+  __shared__ __align__(8) uint64_t s_mma_done[2];   // each MMA issuer's own drain
   __shared__ uint32_t s_tmem;
   __shared__ volatile int s_abort;
   __shared__ int s_par[kMaxNodes];
   __shared__ uint64_t s_anc[kMaxNodes][2];
-  __shared__ int s_pages[kPageChunk];
+  __shared__ int s_pages[2][kPageChunk];   // K / V producer: staged page-table entries
   __shared__ int s_issued[2][S];   // producer: K (0) and V (1) fills issued per stage
 
   pdl_launch_dependents();
@@ -713,7 +713,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(smem_u32(&s_pv_done[x]), 1);
     }
     mbar_init(smem_u32(&s_q_ready), 8);
-    mbar_init(smem_u32(&s_mma_done), 1);
+    mbar_init(smem_u32(&s_mma_done[0]), 1);
+    mbar_init(smem_u32(&s_mma_done[1]), 1);
     s_abort = 0;
     fence_mbar_init();
   }
@@ -740,116 +741,120 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after();
   const uint32_t tmem = s_tmem;
 
-  if (warp == 0) {
-    // ------------------------------------------------------------ TMA producer
-    // K(t) then V(t), each into its own ring; K slots free up as soon as both
-    // S MMAs of their tile are done, V slots after both P.V MMAs
+  if (warp == 0 || warp == 11) {
+    // ----------------------------------------------------------- TMA producers
+    // K (warp 0) and V (warp 11), each into its own ring; K slots free up as
+    // soon as both S MMAs of their tile are done, V slots after both P.V MMAs
+    const int which = warp == 0 ? 0 : 1;
     if (lane == 0) {
-      prefetch_tmap(&tm_k);
-      prefetch_tmap(&tm_v);
-      prefetch_tmap(&tm_tk);
-      prefetch_tmap(&tm_tv);
+      prefetch_tmap(which ? &tm_v : &tm_k);
+      prefetch_tmap(which ? &tm_tv : &tm_tk);
     }
     const uint64_t pol = l2_policy_evict_first();
     int chunk0 = -1;
-    bool ok = true;
-    for (int t = 0; t < it.ntiles && ok; ++t) {
+    bool pok = true;
+    for (int t = 0; t < it.ntiles; ++t) {
       const int stage = t % S;
-      const uint32_t ph = ((t / S) & 1) ^ 1u;
-#pragma unroll
-      for (int which = 0; which < 2; ++which) {
-        uint64_t* empty = which ? &s_v_empty[stage] : &s_k_empty[stage];
-        uint64_t* full = which ? &s_v_full[stage] : &s_k_full[stage];
-        if (!wait_all(empty, ph, budget) || aborted_warp(&s_abort)) {
-          ok = false;
-          break;
-        }
-        const uint32_t dst = base + (which ? G::kVOff : G::kKOff) + stage * G::kKVTile;
-        if (p.page_size != 0 && t < it.nctx)
-          issue_paged_half<D>(p, it, t, dst, smem_u32(full), which ? &tm_v : &tm_k, pol, s_pages,
-                              chunk0, lane);
-        else if (lane == 0)
-          issue_half_tile<D>(p, it, t, dst, smem_u32(full), which ? &tm_v : &tm_k,
-                             which ? &tm_tv : &tm_tk, pol);
-        if (lane == 0) ++s_issued[which][stage];
-        __syncwarp();
+      uint64_t* empty = which ? &s_v_empty[stage] : &s_k_empty[stage];
+      uint64_t* full = which ? &s_v_full[stage] : &s_k_full[stage];
+      if (!wait_all(empty, ((t / S) & 1) ^ 1u, budget) || aborted_warp(&s_abort)) {
+        pok = false;
+        break;
       }
+      const uint32_t dst = base + (which ? G::kVOff : G::kKOff) + stage * G::kKVTile;
+      if (p.page_size != 0 && t < it.nctx)
+        issue_paged_half<D>(p, it, t, dst, smem_u32(full), which ? &tm_v : &tm_k, pol,
+                            s_pages[which], chunk0, lane);
+      else if (lane == 0)
+        issue_half_tile<D>(p, it, t, dst, smem_u32(full), which ? &tm_v : &tm_k,
+                           which ? &tm_tv : &tm_tk, pol);
+      if (lane == 0) ++s_issued[which][stage];
+      __syncwarp();
     }
-    if (!ok && lane == 0) {
+    if (!pok && lane == 0) {
       note_timeout(p.status);
       s_abort = 1;
     }
     // every copy issued has landed before the buffers are reused or left
     if (lane == 0)
-      for (int which = 0; which < 2; ++which)
-        for (int s = 0; s < S; ++s)
-          if (s_issued[which][s] > 0)
-            mbar_wait(smem_u32(which ? &s_v_full[s] : &s_k_full[s]),
-                      static_cast<uint32_t>((s_issued[which][s] - 1) & 1));
+      for (int st = 0; st < S; ++st)
+        if (s_issued[which][st] > 0)
+          mbar_wait(smem_u32(which ? &s_v_full[st] : &s_k_full[st]),
+                    static_cast<uint32_t>((s_issued[which][st] - 1) & 1));
     __syncwarp();
-  } else if (warp == 1) {
-    // --------------------------------------------------------------- MMA issuer
+  } else if (warp == 1 || warp == 10) {
+    // ------------------------------------------------------------ MMA issuers
+    // Two issuing threads, so that the one's barrier waits overlap the other's
+    // MMAs: warp 1 issues S_x(t) = Q_x K(t)^T, warp 10 O_x += P_x(t) V(t).
+    // While tile A's softmax works on key tile t, the tensor cores run
+    // O_B += P_B V(t-1) and S_B(t); while B's works, O_A += P_A V(t) and
+    // S_A(t+1).  Each commit tracks the issuing thread's own MMAs.
     if (lane == 0) {
-      const uint32_t idesc_s = idesc_bf16(kRows, kKeys);         // S = Q K^T
-      const uint32_t idesc_o = idesc_bf16(kRows, D, true);       // O += P V, V MN-major
-      bool mok = mbar_wait(smem_u32(&s_q_ready), 0, budget);
-      if (mok) tc_fence_after();
-      // S_x(t) = Q_x K(t)^T into tile x's S/P columns; they are free once
-      // O_x += P_x V of tile t-1 is done.  The last S of tile t releases K(t).
-      auto issue_s = [&](int x, int t) -> bool {
-        const int stage = t % S;
-        if (!mbar_wait(smem_u32(&s_k_full[stage]), (t / S) & 1, budget) || s_abort) return false;
-        if (t > 0 && (!mbar_wait(smem_u32(&s_pv_done[x]), (t - 1) & 1, budget) || s_abort))
-          return false;
-        tc_fence_after();
-        const uint32_t kst = base + G::kKOff + stage * G::kKVTile;
-        const uint32_t qst = base + G::kQOff + x * G::kQTile;
+      bool mok = true;
+      if (warp == 1) {
+        const uint32_t idesc_s = idesc_bf16(kRows, kKeys);   // S = Q K^T
+        mok = mbar_wait(smem_u32(&s_q_ready), 0, budget);
+        if (mok) tc_fence_after();
+        for (int t = 0; mok && t < it.ntiles; ++t) {
+          const int stage = t % S;
+          mok = mbar_wait(smem_u32(&s_k_full[stage]), (t / S) & 1, budget);
+          for (int x = 0; mok && x < nx; ++x) {
+            // tile x's S/P columns are free once O_x += P_x V of tile t-1 is done
+            if (t > 0) mok = mbar_wait(smem_u32(&s_pv_done[x]), (t - 1) & 1, budget);
+            if (!mok || s_abort) {
+              mok = false;
+              break;
+            }
+            tc_fence_after();
+            const uint32_t kst = base + G::kKOff + stage * G::kKVTile;
+            const uint32_t qst = base + G::kQOff + x * G::kQTile;
 #pragma unroll
-        for (int ks = 0; ks < D / 16; ++ks) {
-          const int h = ks >> 2, kk = ks & 3;
-          tc_mma(tmem + (256u + 128u * static_cast<uint32_t>(x)),
-                 sw128_desc(qst + h * (kRows * 128) + 32 * kk),
-                 sw128_desc(kst + h * (kKeys * 128) + 32 * kk), idesc_s, ks > 0 ? 1u : 0u);
+            for (int ks = 0; ks < D / 16; ++ks) {
+              const int h = ks >> 2, kk = ks & 3;
+              tc_mma(tmem + (256u + 128u * static_cast<uint32_t>(x)),
+                     sw128_desc(qst + h * (kRows * 128) + 32 * kk),
+                     sw128_desc(kst + h * (kKeys * 128) + 32 * kk), idesc_s, ks > 0 ? 1u : 0u);
+            }
+            tc_commit(smem_u32(&s_s_full[x]));
+          }
+          // the last S of tile t releases K(t)
+          if (mok) tc_commit(smem_u32(&s_k_empty[stage]));
         }
-        tc_commit(smem_u32(&s_s_full[x]));
-        if (x == nx - 1) tc_commit(smem_u32(&s_k_empty[stage]));
-        return true;
-      };
-      // O_x += P_x(t) V(t) once tile x's softmax of tile t is done; the last
-      // P.V of tile t releases V(t)
-      auto issue_pv = [&](int x, int t) -> bool {
-        const int stage = t % S;
-        if (!mbar_wait(smem_u32(&s_v_full[stage]), (t / S) & 1, budget) || s_abort) return false;
-        if (!mbar_wait(smem_u32(&s_p_full[x]), t & 1, budget) || s_abort) return false;
-        tc_fence_after();
-        const uint32_t vst = base + G::kVOff + stage * G::kKVTile;
+      } else {
+        const uint32_t idesc_o = idesc_bf16(kRows, D, true);   // O += P V, V MN-major
+        for (int t = 0; mok && t < it.ntiles; ++t) {
+          const int stage = t % S;
+          mok = mbar_wait(smem_u32(&s_v_full[stage]), (t / S) & 1, budget);
+          for (int x = 0; mok && x < nx; ++x) {
+            // O_x += P_x(t) V(t) once tile x's softmax of key tile t is done
+            mok = mbar_wait(smem_u32(&s_p_full[x]), t & 1, budget);
+            if (!mok || s_abort) {
+              mok = false;
+              break;
+            }
+            tc_fence_after();
+            const uint32_t vst = base + G::kVOff + stage * G::kKVTile;
 #pragma unroll
-        for (int kk = 0; kk < kKeys / 16; ++kk)
-          tc_mma_ts(tmem + static_cast<uint32_t>(x * D),
-                    tmem + (256u + 128u * static_cast<uint32_t>(x)) + kk * 8,
-                    sw128_desc_mn(vst + kk * 2048, kKeys * 128, 1024), idesc_o,
-                    (t > 0 || kk > 0) ? 1u : 0u);
-        tc_commit(smem_u32(&s_pv_done[x]));
-        if (x == nx - 1) tc_commit(smem_u32(&s_v_empty[stage]));
-        return true;
-      };
-      // ping-pong: while tile A's softmax works on tile t, the tensor cores
-      // run O_B += P_B V(t-1) and S_B(t); while B's works, O_A += P_A V(t) and
-      // S_A(t+1)
-      for (int x = 0; mok && x < nx; ++x) mok = issue_s(x, 0);
-      for (int t = 0; mok && t < it.ntiles; ++t) {
-        for (int x = 0; mok && x < nx; ++x) {
-          mok = issue_pv(x, t);
-          if (mok && t + 1 < it.ntiles) mok = issue_s(x, t + 1);
+            for (int kk = 0; kk < kKeys / 16; ++kk)
+              tc_mma_ts(tmem + static_cast<uint32_t>(x * D),
+                        tmem + (256u + 128u * static_cast<uint32_t>(x)) + kk * 8,
+                        sw128_desc_mn(vst + kk * 2048, kKeys * 128, 1024), idesc_o,
+                        (t > 0 || kk > 0) ? 1u : 0u);
+            tc_commit(smem_u32(&s_pv_done[x]));
+          }
+          // the last P.V of tile t releases V(t)
+          if (mok) tc_commit(smem_u32(&s_v_empty[stage]));
         }
       }
       if (!mok) {
         note_timeout(p.status);
         s_abort = 1;
       }
-      // every MMA issued above has finished before TMEM or the buffers are reused
-      tc_commit(smem_u32(&s_mma_done));
-      mbar_wait(smem_u32(&s_mma_done), 0);
+      // every MMA this thread issued has finished before TMEM or the buffers
+      // are reused
+      uint64_t* done = &s_mma_done[warp == 1 ? 0 : 1];
+      tc_commit(smem_u32(done));
+      mbar_wait(smem_u32(done), 0);
     }
     __syncwarp();
   } else {
@@ -1078,7 +1083,7 @@ cudaError_t launch_attention_tc(const AttnParams& p, const CUtensorMap& tm_k,
   auto* k = p.D == 64 ? attn_tc_kernel<64> : attn_tc_kernel<128>;
   err = set_smem_attrs(k, smem);
   if (err != cudaSuccess) return err;
-  return launch_pdl(k, grid, dim3(kTcThreads), smem, s, tm_k, tm_v, tm_tk, tm_tv, p);
+  return launch_pdl(k, grid, dim3(kThreads), smem, s, tm_k, tm_v, tm_tk, tm_tv, p);
 }
 
 }  // namespace asd
