@@ -114,10 +114,43 @@ struct Item {
   int ctx, nctx, ntree, ntiles;
 };
 
-__device__ __forceinline__ bool make_item(const AttnParams& p, Item& it) {
+constexpr int kOrderMax = 256;   // batches ordered by work in-kernel (larger ones: index order)
+
+// The sequence of rank r when the B sequences are ordered by decreasing
+// attention work (their context and tree key tiles, ties by index): the
+// hardware dispatches CTAs in blockIdx order, so the longest items start
+// first and the short ones fill the last wave.  Every thread of the CTA calls
+// it (it synchronises the CTA); s_work holds kOrderMax ints.
+__device__ __forceinline__ int sequence_of_rank(const AttnParams& p, int r, int* s_work,
+                                                int* s_b) {
+  if (p.B > kOrderMax) return r;
+  if (threadIdx.x == 0) *s_b = r;
+  for (int q = threadIdx.x; q < p.B; q += blockDim.x) {
+    const int c = min(max(p.ctx_len[q], 0), p.ctx_max);
+    const int n = min(max(p.cu_nodes[q + 1] - p.cu_nodes[q], 0), kMaxNodes);
+    s_work[q] = (c + kKeys - 1) / kKeys + (n + kKeys - 1) / kKeys;
+  }
+  __syncthreads();
+  for (int q = threadIdx.x; q < p.B; q += blockDim.x) {
+    const int w = s_work[q];
+    int rank = 0;
+    for (int j = 0; j < p.B; ++j) {
+      const int v = s_work[j];
+      rank += (v > w || (v == w && j < q)) ? 1 : 0;
+    }
+    if (rank == r) *s_b = q;
+  }
+  __syncthreads();
+  return *s_b;
+}
+
+// blockIdx.y = (r, g): KV head g of the sequence of rank r (sequence_of_rank);
+// blockIdx.x: the item's block of query rows.
+__device__ __forceinline__ bool make_item(const AttnParams& p, Item& it, int* s_work, int* s_b) {
   const int rb = blockIdx.x, bg = blockIdx.y;
-  it.b = bg / p.Hkv;
-  it.g = bg - it.b * p.Hkv;
+  const int r = bg / p.Hkv;
+  it.b = sequence_of_rank(p, r, s_work, s_b);
+  it.g = bg - r * p.Hkv;
   it.s0 = p.cu_nodes[it.b];
   it.n = p.cu_nodes[it.b + 1] - it.s0;
   it.R = it.n * p.G;
@@ -405,8 +438,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   pdl_launch_dependents();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const long long budget = wait_budget(p.status);
+  __shared__ int s_work[kOrderMax];
+  __shared__ int s_seq;
   Item it;
-  if (!make_item(p, it)) {  // no query rows here (uniform over the CTA)
+  if (!make_item(p, it, s_work, &s_seq)) {  // no query rows here (uniform over the CTA)
     pdl_wait();
     return;
   }
@@ -645,10 +680,12 @@ struct PPGeom {
   static constexpr int kBytes = kVOff + kStages * kKVTile;
 };
 
-__device__ __forceinline__ bool make_item_pp(const AttnParams& p, Item& it) {
+__device__ __forceinline__ bool make_item_pp(const AttnParams& p, Item& it, int* s_work,
+                                             int* s_b) {
   const int rb = blockIdx.x, bg = blockIdx.y;
-  it.b = bg / p.Hkv;
-  it.g = bg - it.b * p.Hkv;
+  const int r = bg / p.Hkv;
+  it.b = sequence_of_rank(p, r, s_work, s_b);
+  it.g = bg - r * p.Hkv;
   it.s0 = p.cu_nodes[it.b];
   it.n = p.cu_nodes[it.b + 1] - it.s0;
   it.R = it.n * p.G;
@@ -687,8 +724,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   pdl_launch_dependents();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const long long budget = wait_budget(p.status);
+  __shared__ int s_work[kOrderMax];
+  __shared__ int s_seq;
   Item it;
-  if (!make_item_pp(p, it)) {  // no query rows here (uniform over the CTA)
+  if (!make_item_pp(p, it, s_work, &s_seq)) {  // no query rows here (uniform over the CTA)
     pdl_wait();
     return;
   }
