@@ -345,7 +345,7 @@ constexpr int kWideA = kM * 128;                     // one node tile's k-block:
 constexpr int kWideSlot = kWideG * kWideA + kWideN * 128;   // 64 KB
 constexpr uint32_t kWideTmemCols = kWideG * kWideN;  // 512
 constexpr int kTileGroups = kLmTileN / kLmBoxRows;   // 32-row groups per packed tile
-constexpr int kWideThreads = 320;                    // producer, MMA, two epilogue groups
+constexpr int kWideThreads = 352;                    // producer, 2 MMA issuers, 2 epilogue groups
 
 __device__ __forceinline__ uint32_t cta_rank_in_cluster() {
   uint32_t r;
@@ -431,7 +431,7 @@ __global__ void __launch_bounds__(kWideThreads, 1)
   __shared__ __align__(8) uint64_t s_empty[kWideStages];
   __shared__ __align__(8) uint64_t s_tfull[kWideG];
   __shared__ __align__(8) uint64_t s_tempty[kWideG];
-  __shared__ __align__(8) uint64_t s_mma_done;
+  __shared__ __align__(8) uint64_t s_mma_done[kWideG];   // each MMA issuer's own drain
   __shared__ uint32_t s_tmem;
   __shared__ volatile int s_abort;
   __shared__ int s_pack_bad;
@@ -471,14 +471,14 @@ __global__ void __launch_bounds__(kWideThreads, 1)
   if (threadIdx.x == 0) {
     for (int s = 0; s < kWideStages; ++s) {
       mbar_init(smem_u32(&s_full[s]), 1);
-      mbar_init(smem_u32(&s_empty[s]), CL);      // every CTA of the cluster reads the stage
+      mbar_init(smem_u32(&s_empty[s]), kWideG * CL);   // both issuers of every CTA read it
       s_issued[s] = 0;
     }
     for (int a = 0; a < kWideG; ++a) {
       mbar_init(smem_u32(&s_tfull[a]), 1);
       mbar_init(smem_u32(&s_tempty[a]), 4);
     }
-    mbar_init(smem_u32(&s_mma_done), 1);
+    for (int j = 0; j < kWideG; ++j) mbar_init(smem_u32(&s_mma_done[j]), 1);
     s_abort = 0;
     int bad = 0;
     if (p.w_packed) {
@@ -602,10 +602,14 @@ __global__ void __launch_bounds__(kWideThreads, 1)
       }
     }
     if (!ok && lane == 0) abort_cta();
-  } else if (warp == 1) {
-    // --------------------------------------------------------------- MMA issuer
-    // Accumulator use u (counted over the kernel) goes to TMEM buffer u % 2;
-    // its empty barrier completes once per lap.
+  } else if (warp == 1 || warp == 10) {
+    // ------------------------------------------------------------ MMA issuers
+    // Two issuing threads, one per node tile of the pair (warp 1: tile 0,
+    // warp 10: tile 1), so that the one's barrier waits overlap the other's
+    // MMAs.  Both read every stage and both release it.  Accumulator use u
+    // (counted over the kernel) goes to TMEM buffer u % 2; its empty barrier
+    // completes once per lap.
+    const int j = warp == 1 ? 0 : 1;
     int stage = 0;
     uint32_t ph = 0;
     int used = 0;
@@ -620,6 +624,8 @@ __global__ void __launch_bounds__(kWideThreads, 1)
         if (2 * vt + 1 < voc.ntiles) voc.tile(2 * vt + 1, p.V, q, g0, ng, v0, rows_hi);
         const int ncols = rows_hi > 0 ? kLmTileN + rows_hi : rows_lo;
         const uint32_t idesc = idesc_bf16(kM, (ncols + 15) & ~15);
+        const int u = used + j;
+        const int acc = u % kWideG;
         for (int kb = 0; kb < nkb && ok; ++kb) {
           ok = __shfl_sync(0xffffffffu, mbar_wait(smem_u32(&s_full[stage]), ph, budget), 0);
           if (!ok || s_abort) {
@@ -629,9 +635,7 @@ __global__ void __launch_bounds__(kWideThreads, 1)
           tc_fence_after();
           const uint32_t a_s = base + stage * kWideSlot;
           const uint32_t b_s = a_s + kWideG * kWideA;
-          for (int j = 0; j < gn; ++j) {
-            const int u = used + j;
-            const int acc = u % kWideG;
+          if (j < gn) {
             if (kb == 0) {
               // the epilogue must have drained this buffer's previous tile
               ok = __shfl_sync(
@@ -655,8 +659,8 @@ __global__ void __launch_bounds__(kWideThreads, 1)
             }
             __syncwarp();
           }
-          if (!ok) break;
-          // the stage is free for refilling once every CTA of the cluster has read it
+          // the stage is free for refilling once both issuers of every CTA of
+          // the cluster have read it
           if (lane == 0) {
             if (CL == 2)
               tc_commit_mc(smem_u32(&s_empty[stage]), both);
@@ -676,8 +680,8 @@ __global__ void __launch_bounds__(kWideThreads, 1)
     // every tcgen05 operation of this thread, the commits included, is done
     // before the CTA leaves the cluster
     if (lane == 0) {
-      tc_commit(smem_u32(&s_mma_done));
-      mbar_wait(smem_u32(&s_mma_done), 0);
+      tc_commit(smem_u32(&s_mma_done[j]));
+      mbar_wait(smem_u32(&s_mma_done[j]), 0);
     }
     __syncwarp();
   } else {
