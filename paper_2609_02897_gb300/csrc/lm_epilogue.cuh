@@ -64,8 +64,14 @@ __device__ __forceinline__ void row_chunk(RowState& st, const float (&r)[32], in
   }
   const float nm = -st.m * kLog2e;
   float acc = 0.f;
+  // one special-function-unit instruction per logit (results below 2^-126 of
+  // the running max flush to zero: they cannot move the fp32 sum)
 #pragma unroll
-  for (int j = 0; j < 32; ++j) acc += exp2f(fmaf(x[j], kLog2e, nm));
+  for (int j = 0; j < 32; ++j) {
+    float e;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(e) : "f"(fmaf(x[j], kLog2e, nm)));
+    acc += e;
+  }
   st.s += acc;
   while (st.next_tok < c0 + nvalid) {
     const int jj = st.next_tok - c0;
