@@ -5,13 +5,14 @@
 // fp32 accumulate.
 //
 // Work item (one CTA): 128 query rows of one (sequence, KV head) pair, the
-// whole context.  The rows of a pair are its N nodes times the G query heads
-// that share the KV head, node-major (row r -> node r / G, head g*G + r % G);
-// row r lives in TMEM lane r.  Keys come in tiles of 128, K and V through
-// TMA rings of their own (128-byte swizzle; paged caches one box per page;
-// the tree K/V through a 3D map over [T, Hkv, D]), so a K slot is refilled
-// as soon as its S MMA is done rather than after the tile's P.V; the
-// last tile of a pair holds its tree keys, where a node sees only its
+// whole context; the CTAs take the sequences in decreasing order of work, so
+// the longest items start first.  The rows of a pair are its N nodes times
+// the G query heads that share the KV head, node-major (row r -> node r / G,
+// head g*G + r % G); row r lives in TMEM lane r.  Keys come in tiles of 128,
+// K and V through TMA rings of their own (128-byte swizzle; paged caches one
+// box per page; the tree K/V through a 3D map over [T, Hkv, D]), so a K slot
+// is refilled as soon as its S MMA is done rather than after the tile's P.V;
+// the last tile of a pair holds its tree keys, where a node sees only its
 // ancestors (bitmasks derived here from the parent array).
 //
 //   Q             staged once into shared memory by the softmax warps
@@ -21,10 +22,9 @@
 //   O += P . V    tcgen05.mma, A (= P) from TMEM, V MN-major straight from its
 //                 TMA tile, O in TMEM for the whole item
 //
-// The softmax keeps a
-// per-row reference max m and rescales O only when the running max exceeds m
-// by more than 2^8 in the exp2 domain (P then stays below 2^8 and the result
-// equals that with the exact running max).  S/P is triple-buffered: S of tile
+// The softmax keeps a per-row reference max m and rescales O only when the
+// running max exceeds m by more than 2^8 in the exp2 domain (P then stays
+// below 2^8 and the result equals that with the exact running max).  S/P is triple-buffered: S of tile
 // t+1 is ready when the softmax finishes tile t, and S of tile t+2 does not
 // wait for O += P V of tile t (with two buffers it did, which put the P.V,
 // its commit and the next S on the softmax's path every second tile).
@@ -44,7 +44,7 @@ namespace {
 
 constexpr int kRows = kAttnTcRows;   // query rows per CTA = TMEM lanes
 constexpr int kKeys = kAttnTcKeys;   // keys per tile
-constexpr int kThreads = 384;   // twelve warps (roles below)
+constexpr int kThreads = 384;   // twelve warps (the roles above; the ping-pong form's below)
 constexpr int kSoftmaxThreads = 256;   // eight warps: two per TMEM lane quarter
 constexpr float kRescaleLog2 = 8.f;
 constexpr uint32_t kTmemCols = 512;

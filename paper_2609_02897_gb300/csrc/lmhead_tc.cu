@@ -12,10 +12,12 @@
 // (max, argmax, sum-exp) per node; the tail kernel merges the ranges.
 //
 // A stage holds two k-blocks (128 hidden elements) of a 128-row vocabulary
-// tile (W, 32 KB, in 64-row TMA boxes) and of the node tile (hidden states,
-// a_rows rows).  Reading 256 contiguous bytes of each weight row per stage,
-// in few large boxes, streams W from HBM markedly faster than one k-block of
-// a 256-row tile per stage.
+// tile (W, 32 KB: one contiguous bulk copy from the packed weight, or 64-row
+// TMA boxes from [V, K] rows) and of the node tile (hidden states, a_rows
+// rows).  Reading 256 contiguous bytes of each weight row per stage streams W
+// from HBM markedly faster than one k-block of a 256-row tile per stage, and
+// the packed order, where every SM's range is one contiguous run, faster
+// still.
 //
 // Warp roles (192 threads): warp 0 TMA producer, warp 1 TMEM allocator and
 // MMA issuer, warps 2-5 epilogue (TMEM lane quarters 2, 3, 0, 1).
@@ -333,18 +335,20 @@ __global__ void __launch_bounds__(192, 1)
 // range and writes one partial per range, so the statistics are those of
 // CTAs that own one range each, bit for bit.
 //
-// Warp roles (320 threads): warp 0 TMA producer, warp 1 TMEM allocator and MMA
-// issuer, warps 2-5 and 6-9 two epilogue groups; group g drains the
-// accumulator of the pair's node tile g, so that both accumulators of a
-// vocabulary tile are drained at once and the MMAs of the next tile wait for
-// one drain instead of two.
+// Warp roles (352 threads): warp 0 TMA producer, warp 1 TMEM allocator and
+// MMA issuer for node tile 0 of every pair, warp 10 MMA issuer for node tile
+// 1 (two issuing threads: a barrier wait costs its thread a few hundred
+// cycles, and one thread's waits then overlap the other's MMAs), warps 2-5
+// and 6-9 two epilogue groups; group g drains the accumulator of the pair's
+// node tile g, so that both accumulators of a vocabulary tile are drained at
+// once and the MMAs of the next tile wait for one drain instead of two.
 constexpr int kWideN = 2 * kLmTileN;                 // vocabulary rows per MMA
 constexpr int kWideG = 2;                            // node tiles per W stage and CTA
 constexpr int kWideStages = 3;
 constexpr int kWideA = kM * 128;                     // one node tile's k-block: 16 KB
 constexpr int kWideSlot = kWideG * kWideA + kWideN * 128;   // 64 KB
 constexpr uint32_t kWideTmemCols = kWideG * kWideN;  // 512
-constexpr int kTileGroups = kLmTileN / kLmBoxRows;   // 32-row groups per packed tile
+constexpr int kTileGroups = kLmTileN / kLmBoxRows;   // range groups per packed tile
 constexpr int kWideThreads = 352;                    // producer, 2 MMA issuers, 2 epilogue groups
 
 __device__ __forceinline__ uint32_t cta_rank_in_cluster() {
