@@ -908,14 +908,17 @@ cudaError_t launch_wide(const LmParams& p, const LmMaps& maps, cudaStream_t s) {
 int lmhead_bf16_variant(const LmParams& p) {
   if (p.T <= kM && !p.t_dev) return 1;
   // several node tiles, or a row count known on the device only: the wide
-  // kernel (full 128-row node boxes).  Clusters of two pay when every CTA has
-  // at least two rounds of node pairs (the CTAs of a cluster move in lock
-  // step; with one round the coupling costs more than the halved W traffic
-  // saves), and when the ranges pair up.  Their W multicast reads this GPU's
-  // own memory only: a weight elsewhere (host or another device) runs
-  // unclustered.
+  // kernel (full 128-row node boxes).  Clusters of two halve the W traffic
+  // (each W stage is read once per cluster) and move their CTAs in lock step
+  // through the rounds of node pairs, so they pay unless that lock step leaves
+  // one CTA idle for a large share of the work: with three pairs the CTA
+  // without a pair in the second round idles for half of it (measured with
+  // two MMA-issuing threads: two pairs 430 -> 393 us on the Qwen3-8B B8
+  // workload, four and more pairs 10 % faster).  The ranges must pair up, and
+  // the W multicast reads this GPU's own memory only: a weight elsewhere
+  // (host or another device) runs unclustered.
   const int pairs = (p.T + kWideG * kM - 1) / (kWideG * kM);
-  return (p.g_lm % 2 == 0 && !p.t_dev && pairs >= 4 && p.w_local) ? 3 : 2;
+  return (p.g_lm % 2 == 0 && !p.t_dev && (pairs == 2 || pairs >= 4) && p.w_local) ? 3 : 2;
 }
 
 cudaError_t launch_lmhead_bf16(const LmParams& p, const LmMaps& maps, cudaStream_t s) {

@@ -32,8 +32,11 @@ def test_cluster_form_only_for_a_weight_on_this_gpu(dev):
     assert asd.asd_lm_head_variant(dims, wl.T, w_dev) == (3 if ranges % 2 == 0 else 2)
     assert asd.asd_lm_head_variant(dims, wl.T, w_pinned) == 2
     assert asd.asd_lm_head_variant(dims, wl.T, w_pageable) == 2
-    # three tile pairs or fewer: unclustered whatever the weight
+    # two tile pairs: clustered (with pairing ranges); three: unclustered (one
+    # CTA of a cluster would idle through the second round)
+    assert asd.asd_lm_head_variant(dims, 512, w_dev) == (3 if ranges % 2 == 0 else 2)
     assert asd.asd_lm_head_variant(dims, 768, w_dev) == 2
+    assert asd.asd_lm_head_variant(dims, 256, w_dev) == 2
     # the lazy schedule's levels run the wide kernel unclustered
     dims.lm_head_schedule = asd.ASD_LM_LAZY_LEVELS
     assert asd.asd_lm_head_variant(dims, wl.T, w_dev) == 2
