@@ -303,8 +303,8 @@ int32_t asd_abi_version(void);
  * runs (a diagnostic query; no counterpart in the paper; nothing is
  * launched): 1 the weight-streaming tensor-core kernel (up to 128 nodes),
  * 2 the wide kernel (more nodes, or a level of the lazy schedule), 3 the wide
- * kernel in clusters of two SMs that multicast W between them (more than
- * three pairs of 128-node tiles and an even range count), 4 the fp32 kernel,
+ * kernel in clusters of two SMs that multicast W between them (two pairs of
+ * 128-node tiles, or four and more, and an even range count), 4 the fp32 kernel,
  * 0 for invalid arguments.  The clustered form multicasts from the calling
  * GPU's own memory only: when w_lm is not device memory of the current device
  * the call runs form 2.
