@@ -297,6 +297,7 @@ __device__ __forceinline__ bool softmax_role(const AttnParams& p, const Item& it
   const float c = p.scale_log2;
   float m_ref = -INFINITY, l = 0.f;
   bool ok = true, bad = false;
+  bool s_seen = false;   // S of tile t already seen complete (probed during tile t-1)
   for (int t = 0; t < it.ntiles; ++t) {
     const int b = t % kSBufs, e = t & 1;
     const uint32_t sb = lane_base + kSCol0 + b * kKeys;
@@ -305,8 +306,8 @@ __device__ __forceinline__ bool softmax_role(const AttnParams& p, const Item& it
     const int valid = min(kKeys, (tree ? it.n : it.ctx) - key0);
     float x[64];
     float mt = -INFINITY;
-    const bool here =
-        !bad && wait_all(&s_full[b], (t / kSBufs) & 1, budget) && !aborted_warp(s_abort);
+    const bool here = !bad && (s_seen || wait_all(&s_full[b], (t / kSBufs) & 1, budget)) &&
+                      !aborted_warp(s_abort);
     if (here) {
       tc_fence_after();
       tmem_ld64(sb + 64 * hf, x);
@@ -324,6 +325,13 @@ __device__ __forceinline__ bool softmax_role(const AttnParams& p, const Item& it
       for (int k = 0; k < 64; ++k) mt = fmaxf(mt, x[k]);
       s_mx[e][hf][row] = mt;
     }
+    // probe S of the next tile now (non-blocking), so that the barrier's
+    // latency passes under this tile's exponentials; once complete, that
+    // phase stays complete until this warp has consumed the tile
+    s_seen = __all_sync(0xffffffffu,
+                        t + 1 < it.ntiles &&
+                            mbar_test_wait(smem_u32(&s_full[(t + 1) % kSBufs]),
+                                           static_cast<uint32_t>(((t + 1) / kSBufs) & 1)));
     // every softmax warp decides together whether to go on (no warp may be
     // left waiting at a barrier), and the partial maxima become visible
     ok = softmax_all(here);
