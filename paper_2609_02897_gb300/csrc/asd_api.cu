@@ -61,6 +61,23 @@ bool make_tree_tmap_bf16(CUtensorMap* tm, const void* base, uint64_t d, uint64_t
              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// q [T, Hq, D] bf16 as a 3D map {D, Hq, T}: a box of 64 columns x G heads x
+// kAttnTcRows / G nodes lands as the kAttnTcRows query rows of one KV head's
+// block (node-major, head-minor), 128-byte swizzled.
+bool make_q_tmap_bf16(CUtensorMap* tm, const void* base, uint64_t d, uint64_t hq, uint64_t t,
+                      int g) {
+  EncodeTiledFn enc = encode_fn();
+  if (!enc || g < 1 || kAttnTcRows % g != 0) return false;
+  const cuuint64_t dims[3] = {d, hq, t};
+  const cuuint64_t strides[2] = {d * 2, hq * d * 2};
+  const cuuint32_t box[3] = {64, static_cast<cuuint32_t>(g),
+                             static_cast<cuuint32_t>(kAttnTcRows / g)};
+  const cuuint32_t estr[3] = {1, 1, 1};
+  return enc(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box,
+             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 }  // namespace
 
 int asd::lm_ranges(int vocab, int nsm) {
@@ -260,7 +277,7 @@ asd_status run_attention(const Ctx& c, const void* q, const void* k_cache, const
   a.scale_log2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(d.head_dim)));
   cudaError_t err;
   if (c.L.attn_tc) {
-    CUtensorMap tk, tv, ttk, ttv;
+    CUtensorMap tk, tv, ttk, ttv, tq;
     uint64_t rows;
     uint32_t box_rows;
     if (d.page_size == 0) {
@@ -276,7 +293,14 @@ asd_status run_attention(const Ctx& c, const void* q, const void* k_cache, const
         !make_tree_tmap_bf16(&ttk, tree_k, d.head_dim, d.num_kv_heads, c.T, kAttnTcKeys) ||
         !make_tree_tmap_bf16(&ttv, tree_v, d.head_dim, d.num_kv_heads, c.T, kAttnTcKeys))
       return ASD_ERR_CUDA;
-    err = launch_attention_tc(a, tk, tv, ttk, ttv, c.L.attn_tc == 2, c.st);
+    // the single-tile kernel loads the query tile by TMA where G divides its
+    // 128 rows (otherwise its softmax warps stage it; tq then goes unused)
+    tq = ttk;
+    if (c.L.attn_tc == 1 && attention_q_tma_ok(a.G)) {
+      if (!make_q_tmap_bf16(&tq, q, d.head_dim, d.num_q_heads, c.T, a.G)) return ASD_ERR_CUDA;
+      a.q_tma = 1;
+    }
+    err = launch_attention_tc(a, tk, tv, ttk, ttv, tq, c.L.attn_tc == 2, c.st);
   } else if (d.dtype == ASD_BF16) {
     CUtensorMap tk, tv;
     uint64_t rows;

@@ -244,6 +244,23 @@ __device__ __forceinline__ void issue_paged_half(const AttnParams& p, const Item
   __syncwarp();
 }
 
+// The query tile of an item by TMA (p.q_tma): a 3D map over q [T, Hq, D]
+// with boxes of 64 columns x G heads x 128/G nodes lands as the item's 128
+// rows (node-major, head-minor, as grow_of numbers them), 128-byte swizzled;
+// rows past the item's hold the next nodes' queries (or zeros past T), which
+// no output row reads.
+template <int D>
+__device__ __forceinline__ void issue_q_tile(const AttnParams& p, const Item& it, uint32_t q_s,
+                                             uint32_t bar, const CUtensorMap* tm_q,
+                                             uint64_t pol) {
+  using G = TcGeom<D>;
+  mbar_expect_tx(bar, static_cast<uint32_t>(G::kNH * kRows * 128));
+#pragma unroll
+  for (int h = 0; h < G::kNH; ++h)
+    tma_load_3d(q_s + h * (kRows * 128), tm_q, bar, h * 64, it.g * p.G, it.s0 + it.r0 / p.G,
+                pol);
+}
+
 // Softmax warps (eight): warp w handles TMEM lane quarter w % 4 (its 32 query
 // rows, one thread per row) and half h = (w - 2) / 4 of every tile's 128 keys.
 // Per tile: read its 64 S columns, mask, exchange the row's partial max with
@@ -271,7 +288,8 @@ __device__ __forceinline__ bool softmax_role(const AttnParams& p, const Item& it
 
   // this half of the row's query (16-byte chunks [hf D/16, (hf+1) D/16)) ->
   // shared memory, 128-byte swizzled like a TMA tile; zeros past nrows
-  {
+  // (unless the query tile comes by TMA)
+  if (!p.q_tma) {
     const bool mine = row < it.nrows;
     const uint4* qg = reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(p.q) +
                                                      (mine ? grow_of(p, it, row) : 0) * D);
@@ -284,9 +302,11 @@ __device__ __forceinline__ bool softmax_role(const AttnParams& p, const Item& it
                                 (((c & 7) ^ (row & 7)) << 4)) = v;
     }
   }
-  fence_proxy_async();   // the tensor cores read these rows
-  __syncwarp();
-  if (lane == 0) mbar_arrive(smem_u32(q_ready));
+  if (!p.q_tma) {
+    fence_proxy_async();   // the tensor cores read these rows
+    __syncwarp();
+    if (lane == 0) mbar_arrive(smem_u32(q_ready));
+  }
 
   uint64_t alo = 0, ahi = 0;
   if (row < it.nrows) {
@@ -423,7 +443,8 @@ template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_v,
                    const __grid_constant__ CUtensorMap tm_tk,
-                   const __grid_constant__ CUtensorMap tm_tv, const AttnParams p) {
+                   const __grid_constant__ CUtensorMap tm_tv,
+                   const __grid_constant__ CUtensorMap tm_q, const AttnParams p) {
   using G = TcGeom<D>;
   extern __shared__ uint8_t smem_raw[];
   constexpr int KS = G::kKStages, VS = G::kVStages;
@@ -476,11 +497,31 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(smem_u32(&s_p_full[b]), kSoftmaxThreads / 32);
       mbar_init(smem_u32(&s_pv_done[b]), 1);
     }
-    mbar_init(smem_u32(&s_q_ready), kSoftmaxThreads / 32);
+    // the query: one TMA (p.q_tma) or the eight softmax warps' stores
+    mbar_init(smem_u32(&s_q_ready), p.q_tma ? 1 : kSoftmaxThreads / 32);
     mbar_init(smem_u32(&s_mma_done[0]), 1);
     mbar_init(smem_u32(&s_mma_done[1]), 1);
     s_abort = 0;
     fence_mbar_init();
+    // The item's first copies go out before the rest of the set-up: its
+    // query tile (TMA form), then the first fill of both rings on a
+    // contiguous cache (the producers go on from there).  What the first S
+    // MMA waits for then lands while the CTA allocates TMEM and builds the
+    // ancestor masks.
+    const uint64_t pol = l2_policy_evict_first();
+    if (p.q_tma) issue_q_tile<D>(p, it, q_s, smem_u32(&s_q_ready), &tm_q, pol);
+    if (p.page_size == 0) {
+      for (int t = 0; t < KS && t < it.ntiles; ++t) {
+        issue_half_tile<D>(p, it, t, k_s0 + t * G::kTileBytes, smem_u32(&s_k_full[t]), &tm_k,
+                           &tm_tk, pol);
+        s_issued[0][t] = 1;
+        if (t < VS) {
+          issue_half_tile<D>(p, it, t, v_s0 + t * G::kTileBytes, smem_u32(&s_v_full[t]), &tm_v,
+                             &tm_tv, pol);
+          s_issued[1][t] = 1;
+        }
+      }
+    }
   }
   if (warp == 1) {
     tmem_alloc(smem_u32(&s_tmem), kTmemCols);
@@ -524,7 +565,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint64_t pol = l2_policy_evict_first();
     int chunk0 = -1;
     bool pok = true;
-    for (int t = 0; pok && t < it.ntiles; ++t) {
+    // on a contiguous cache the first fill of the ring went out with the set-up
+    for (int t = p.page_size == 0 ? ns : 0; pok && t < it.ntiles; ++t) {
       const int stage = t % ns;
       uint64_t* empty = which ? &s_v_empty[stage] : &s_k_empty[stage];
       uint64_t* full = which ? &s_v_full[stage] : &s_k_full[stage];
@@ -547,11 +589,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       s_abort = 1;
     }
     // every copy issued has landed before the buffers are reused or left
-    if (lane == 0)
+    // (the query tile's too, which a wait that gave up may have left in flight)
+    if (lane == 0) {
       for (int st = 0; st < ns; ++st)
         if (s_issued[which][st] > 0)
           mbar_wait(smem_u32(which ? &s_v_full[st] : &s_k_full[st]),
                     static_cast<uint32_t>((s_issued[which][st] - 1) & 1));
+      if (which == 0 && p.q_tma) mbar_wait(smem_u32(&s_q_ready), 0);
+    }
     __syncwarp();
   } else if (warp == 1 || warp == 10) {
     // ------------------------------------------------------------ MMA issuers
@@ -1113,9 +1158,12 @@ bool attention_pingpong(int batch, int num_kv_heads, int G, int total_nodes, int
   return batch > 0 && items >= 2LL * nsm;
 }
 
+bool attention_q_tma_ok(int G) { return G >= 1 && kRows % G == 0; }
+
 cudaError_t launch_attention_tc(const AttnParams& p, const CUtensorMap& tm_k,
                                 const CUtensorMap& tm_v, const CUtensorMap& tm_tk,
-                                const CUtensorMap& tm_tv, bool pingpong, cudaStream_t s) {
+                                const CUtensorMap& tm_tv, const CUtensorMap& tm_q, bool pingpong,
+                                cudaStream_t s) {
   const size_t smem = attention_tc_smem_bytes(p.D, pingpong);
   if (p.D != 64 && p.D != 128) return cudaErrorInvalidValue;
   cudaError_t err;
@@ -1130,7 +1178,7 @@ cudaError_t launch_attention_tc(const AttnParams& p, const CUtensorMap& tm_k,
   auto* k = p.D == 64 ? attn_tc_kernel<64> : attn_tc_kernel<128>;
   err = set_smem_attrs(k, smem);
   if (err != cudaSuccess) return err;
-  return launch_pdl(k, grid, dim3(kThreads), smem, s, tm_k, tm_v, tm_tk, tm_tv, p);
+  return launch_pdl(k, grid, dim3(kThreads), smem, s, tm_k, tm_v, tm_tk, tm_tv, tm_q, p);
 }
 
 }  // namespace asd

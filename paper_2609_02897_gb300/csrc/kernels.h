@@ -75,6 +75,7 @@ struct AttnParams {
   int ctx_max, page_size, pages_per_seq, num_pages;
   int n_splits, split_len, n_parts, max_nodes;
   float scale_log2;         // log2(e) / sqrt(D)
+  int q_tma;                // tensor-core single-tile kernel: the query tile by TMA (tm_q)
 };
 // bf16 path: tensor-core (mma.sync) split-KV kernel fed by TMA; tm_k / tm_v are
 // 2D tensor maps over the context cache rows (box 64 columns x
@@ -90,7 +91,9 @@ int attention_keys_per_tile();   // context keys per K/V tile = TMA box rows
 // sequence x KV head), the whole context, no splits (p.n_parts == 1).  tm_k /
 // tm_v: 2D maps over the cache rows with boxes of 64 columns x
 // min(kAttnTcKeys, rows per page) rows; tm_tk / tm_tv: 3D maps over the tree
-// K/V [T, Hkv, D] with boxes of 64 columns x 1 head x kAttnTcKeys nodes.
+// K/V [T, Hkv, D] with boxes of 64 columns x 1 head x kAttnTcKeys nodes;
+// tm_q (single-tile kernel with p.q_tma, attention_q_tma_ok(G)): a 3D map over
+// q [T, Hq, D] with boxes of 64 columns x G heads x kAttnTcRows / G nodes.
 // pingpong: the two-query-tile form (256 rows per CTA: one tile's MMAs run
 // during the other's softmax), chosen by attention_pingpong() when its items
 // fill at least two waves of CTAs.
@@ -98,9 +101,11 @@ constexpr int kAttnTcRows = 128;   // query rows per CTA (per tile of the ping-p
 constexpr int kAttnTcKeys = 128;   // keys per tile
 size_t attention_tc_smem_bytes(int head_dim, bool pingpong);
 bool attention_pingpong(int batch, int num_kv_heads, int G, int total_nodes, int nsm);
+bool attention_q_tma_ok(int G);   // G divides kAttnTcRows: a query box of whole nodes
 cudaError_t launch_attention_tc(const AttnParams& p, const CUtensorMap& tm_k,
                                 const CUtensorMap& tm_v, const CUtensorMap& tm_tk,
-                                const CUtensorMap& tm_tv, bool pingpong, cudaStream_t s);
+                                const CUtensorMap& tm_tv, const CUtensorMap& tm_q, bool pingpong,
+                                cudaStream_t s);
 
 // -------------------------------------------------------------------- LM head
 struct LmParams {
