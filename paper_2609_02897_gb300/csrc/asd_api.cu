@@ -293,10 +293,10 @@ asd_status run_attention(const Ctx& c, const void* q, const void* k_cache, const
         !make_tree_tmap_bf16(&ttk, tree_k, d.head_dim, d.num_kv_heads, c.T, kAttnTcKeys) ||
         !make_tree_tmap_bf16(&ttv, tree_v, d.head_dim, d.num_kv_heads, c.T, kAttnTcKeys))
       return ASD_ERR_CUDA;
-    // the single-tile kernel loads the query tile by TMA where G divides its
-    // 128 rows (otherwise its softmax warps stage it; tq then goes unused)
+    // the tensor-core kernels load the query tiles by TMA where G divides
+    // their 128 rows (otherwise the softmax warps stage them; tq goes unused)
     tq = ttk;
-    if (c.L.attn_tc == 1 && attention_q_tma_ok(a.G)) {
+    if (attention_q_tma_ok(a.G)) {
       if (!make_q_tmap_bf16(&tq, q, d.head_dim, d.num_q_heads, c.T, a.G)) return ASD_ERR_CUDA;
       a.q_tma = 1;
     }

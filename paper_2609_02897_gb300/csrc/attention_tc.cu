@@ -757,7 +757,8 @@ template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_pp_kernel(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_v,
                    const __grid_constant__ CUtensorMap tm_tk,
-                   const __grid_constant__ CUtensorMap tm_tv, const AttnParams p) {
+                   const __grid_constant__ CUtensorMap tm_tv,
+                   const __grid_constant__ CUtensorMap tm_q, const AttnParams p) {
   using G = PPGeom<D>;
   constexpr int S = G::kStages;
   extern __shared__ uint8_t smem_raw[];
@@ -804,11 +805,23 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(smem_u32(&s_p_full[x]), 4);
       mbar_init(smem_u32(&s_pv_done[x]), 1);
     }
-    mbar_init(smem_u32(&s_q_ready), 8);
+    // the query tiles: one TMA per present tile (p.q_tma), issued before the
+    // rest of the set-up, or the eight softmax warps' stores
+    mbar_init(smem_u32(&s_q_ready), p.q_tma ? 1 : 8);
     mbar_init(smem_u32(&s_mma_done[0]), 1);
     mbar_init(smem_u32(&s_mma_done[1]), 1);
     s_abort = 0;
     fence_mbar_init();
+    if (p.q_tma) {
+      const uint64_t pol = l2_policy_evict_first();
+      const uint32_t bar = smem_u32(&s_q_ready);
+      mbar_expect_tx(bar, static_cast<uint32_t>(nx * G::kQTile));
+      for (int x = 0; x < nx; ++x)
+#pragma unroll
+        for (int h = 0; h < G::kNH; ++h)
+          tma_load_3d(base + G::kQOff + x * G::kQTile + h * (kRows * 128), &tm_q, bar, h * 64,
+                      it.g * p.G, it.s0 + (it.r0 + x * kRows) / p.G, pol);
+    }
   }
   if (warp == 1) {
     tmem_alloc(smem_u32(&s_tmem), kTmemCols);
@@ -868,11 +881,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       s_abort = 1;
     }
     // every copy issued has landed before the buffers are reused or left
-    if (lane == 0)
+    // (the query tiles' too, which a wait that gave up may have left in flight)
+    if (lane == 0) {
       for (int st = 0; st < S; ++st)
         if (s_issued[which][st] > 0)
           mbar_wait(smem_u32(which ? &s_v_full[st] : &s_k_full[st]),
                     static_cast<uint32_t>((s_issued[which][st] - 1) & 1));
+      if (which == 0 && p.q_tma) mbar_wait(smem_u32(&s_q_ready), 0);
+    }
     __syncwarp();
   } else if (warp == 1 || warp == 10) {
     // ------------------------------------------------------------ MMA issuers
@@ -958,7 +974,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t lane_base = tmem + (static_cast<uint32_t>((warp & 3) * 32) << 16);
     const uint32_t sb = lane_base + (256u + 128u * static_cast<uint32_t>(x));
     // the row's query -> shared memory, 128-byte swizzled like a TMA tile
-    {
+    // (unless the query tiles come by TMA)
+    if (!p.q_tma) {
       const int q_row = it.r0 + rr;
       const int node = q_row / p.G;
       const uint4* qg = reinterpret_cast<const uint4*>(
@@ -1172,7 +1189,7 @@ cudaError_t launch_attention_tc(const AttnParams& p, const CUtensorMap& tm_k,
     auto* k = p.D == 64 ? attn_pp_kernel<64> : attn_pp_kernel<128>;
     err = set_smem_attrs(k, smem);
     if (err != cudaSuccess) return err;
-    return launch_pdl(k, grid, dim3(kThreads), smem, s, tm_k, tm_v, tm_tk, tm_tv, p);
+    return launch_pdl(k, grid, dim3(kThreads), smem, s, tm_k, tm_v, tm_tk, tm_tv, tm_q, p);
   }
   const dim3 grid((p.max_nodes * p.G + kRows - 1) / kRows, p.B * p.Hkv, 1);
   auto* k = p.D == 64 ? attn_tc_kernel<64> : attn_tc_kernel<128>;

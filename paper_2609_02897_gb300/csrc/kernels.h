@@ -75,7 +75,7 @@ struct AttnParams {
   int ctx_max, page_size, pages_per_seq, num_pages;
   int n_splits, split_len, n_parts, max_nodes;
   float scale_log2;         // log2(e) / sqrt(D)
-  int q_tma;                // tensor-core single-tile kernel: the query tile by TMA (tm_q)
+  int q_tma;                // tensor-core kernels: the query tiles by TMA (tm_q)
 };
 // bf16 path: tensor-core (mma.sync) split-KV kernel fed by TMA; tm_k / tm_v are
 // 2D tensor maps over the context cache rows (box 64 columns x
@@ -92,7 +92,7 @@ int attention_keys_per_tile();   // context keys per K/V tile = TMA box rows
 // tm_v: 2D maps over the cache rows with boxes of 64 columns x
 // min(kAttnTcKeys, rows per page) rows; tm_tk / tm_tv: 3D maps over the tree
 // K/V [T, Hkv, D] with boxes of 64 columns x 1 head x kAttnTcKeys nodes;
-// tm_q (single-tile kernel with p.q_tma, attention_q_tma_ok(G)): a 3D map over
+// tm_q (with p.q_tma, where attention_q_tma_ok(G)): a 3D map over
 // q [T, Hq, D] with boxes of 64 columns x G heads x kAttnTcRows / G nodes.
 // pingpong: the two-query-tile form (256 rows per CTA: one tile's MMAs run
 // during the other's softmax), chosen by attention_pingpong() when its items
