@@ -29,7 +29,8 @@
  *    ASD_MAX_TREE_NODES nodes per sequence.
  *  - Row-major layouts, innermost dimension last.  Element type of q, caches,
  *    tree K/V, hidden, W and the attention output: dims->dtype (fp32 or bf16).
- *    Tensors read through TMA (caches, hidden, W) must be 16-byte aligned.
+ *    Tensors read through TMA (q, caches, tree K/V, hidden, W) must be
+ *    16-byte aligned; the calls check it and return ASD_ERR_INVALID_ARG.
  *  - tau is the paper's margin threshold kappa (Eq. 1 and the rule after it),
  *    0 < tau <= 1.  The rule is evaluated as l_draft - row_max >= ln(tau) with
  *    ln(tau) computed on the host in double precision.
