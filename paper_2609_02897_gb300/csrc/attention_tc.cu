@@ -15,7 +15,8 @@
 // the last tile of a pair holds its tree keys, where a node sees only its
 // ancestors (bitmasks derived here from the parent array).
 //
-//   Q             staged once into shared memory by the softmax warps
+//   Q             loaded once into shared memory by one TMA (G dividing 128:
+//                 boxes of G heads x 128/G nodes), else by the softmax warps
 //   S = Q . K^T   tcgen05.mma, Q and K K-major in shared memory
 //   P = exp2(S*c - m), per row by the thread that owns the row, written back
 //                 over the tile's S columns as bf16 pairs
@@ -710,7 +711,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 // both: S_A = Q_A.K^T and S_B = Q_B.K^T, then O_A += P_A.V and O_B += P_B.V, so
 // the MMAs of one tile run while the other tile's softmax works, and a K/V
 // byte feeds twice the products.  Q stays in shared memory (both tiles, 128-byte
-// swizzled, written by the softmax threads); TMEM holds O_A [0, D),
+// swizzled, by TMA or written by the softmax threads); TMEM holds O_A [0, D),
 // O_B [D, 2D) and S/P_A [256, 384), S/P_B [384, 512).  K and V come through
 // separate rings with their own barriers, so a K slot is refilled as soon as
 // both S MMAs have read it.  Warps: 0 K producer, 1 S-MMA issuer (lane 0),
